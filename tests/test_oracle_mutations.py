@@ -1,0 +1,66 @@
+"""Plant plausible mistakes in copies of the CPU oracle and check that the pins
+catch every one of them (the planted copies live in a temporary directory)."""
+import os
+import shutil
+import subprocess
+
+import pytest
+
+from oracle import oracle as O
+from tests import _pins
+
+SRC = os.path.join(os.path.dirname(O.__file__), "gba_oracle.c")
+
+# (name, original text, planted text, occurrence index to replace)
+MUTATIONS = [
+    ("dense-boundary-strict", "f[m] = (s <= (int64_t)rule->iota)", "f[m] = (s < (int64_t)rule->iota)", 0),
+    ("row-boundary-strict", "int keep = (s <= (int64_t)rule->iota);",
+     "int keep = (s < (int64_t)rule->iota);", 0),
+    ("dense-divides-by-kept", "float g = gsum / (float)M;",
+     "float g = gsum / (float)(st.msgs_kept > 0 ? st.msgs_kept : 1);", 0),
+    ("row-divides-by-kept-messages", "int64_t denom = cnt[r];", "int64_t denom = cnt_kept[r];", 0),
+    ("row-uses-message-staleness", "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k;",
+     "int64_t ref = k;", 0),
+    ("tag-not-compared", "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k;",
+     "int64_t ref = tokens[m];", 0),
+    ("adagrad-sign", "*w = *w - step / den;", "*w = *w + step / den;", 0),
+    ("adagrad-old-accumulator", "float den = sqrtf(an);", "float den = sqrtf(*a);", 0),
+    ("row-transposed", "S[r * d + j] += (double)gm[i * d + j];",
+     "S[r * d + j] += (double)gm[j * nm + i];", 0),
+    ("no-skip-of-dropped-rows", "if (kept_occ[r] == 0) continue;", "if (kept_occ[r] < 0) continue;", 0),
+    ("adam-step-count", "int64_t t_step = k + 1;", "int64_t t_step = k + 2;", 0),
+    ("counts-occurrences", "if (last_m[r] != m) {", "if (1) {", 0),
+    ("adam-moment-order", "float mn = o->beta1 * *m + c1 * g;", "float mn = c1 * *m + o->beta1 * g;", 0),
+    ("dense-drop-ignored", "if (f[m]) S += (double)dense_grads[m][e];",
+     "S += (double)dense_grads[m][e];", 0),
+    ("init-scale", "return (float)top * 0x1p-27f;", "return (float)top * 0x1p-26f;", 0),
+    ("fifo-overshoot", "if (acc >= G) return i + 1;", "if (acc > G) return i + 1;", 0),
+]
+
+
+def _plant(tmp_path, name, old, new, occ):
+    src = open(SRC).read()
+    idx = -1
+    for _ in range(occ + 1):
+        idx = src.index(old, idx + 1)
+    planted = src[:idx] + new + src[idx + len(old):]
+    c = tmp_path / f"{name}.c"
+    so = tmp_path / f"{name}.so"
+    c.write_text(planted)
+    subprocess.check_call(["gcc", "-O2", "-std=c11", "-ffp-contract=off", "-shared", "-fPIC",
+                           "-o", str(so), str(c), "-lm"])
+    return O.load(str(so))
+
+
+@pytest.mark.parametrize("mut", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_pins_catch_planted_mistake(tmp_path, mut):
+    if shutil.which("gcc") is None:
+        pytest.skip("gcc missing")
+    L = _plant(tmp_path, *mut)
+    caught = []
+    for pin in _pins.ALL_PINS + [_pins.pin_init_published]:
+        try:
+            pin(L)
+        except (AssertionError, ValueError, FloatingPointError):
+            caught.append(pin.__name__)
+    assert caught, f"no pin caught the planted mistake {mut[0]}"
