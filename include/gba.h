@@ -1,0 +1,251 @@
+/*
+ * gba.h - C ABI of libgba: the GBA aggregate-and-apply step on one GB300 GPU.
+ *
+ * GBA (Global Batch gradients Aggregation, arXiv 2205.11048) keeps the global
+ * batch of synchronous training while workers push asynchronously: the
+ * parameter server buffers (gradient, token) messages until the buffered local
+ * batches reach the global batch, excludes gradients whose token staleness
+ * exceeds a threshold (Sec. 4.1, Eq. (1)), and applies the aggregate once per
+ * global step (Alg. 2, push responding threads).
+ *
+ * Conventions for every entry point:
+ *  - No exception crosses this ABI.  Functions return a gba_status (or a
+ *    documented integer); GBA_OK is 0, errors are negative.
+ *  - A handle is used by one host thread at a time.
+ *  - All GPU work of a handle is issued on the stream given to gba_create, in
+ *    submission order; results are visible to work ordered after it on that
+ *    stream, or after gba_sync.
+ *  - Device errors found by a kernel (an id out of range, a bounded wait that
+ *    gave up) are latched: the next gba_try_apply or gba_sync returns the code
+ *    and the handle refuses further steps with GBA_E_STATE.
+ */
+#ifndef GBA_H_
+#define GBA_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gba_handle gba_handle; /* opaque, owned by the library */
+
+typedef enum {
+  GBA_OK = 0,
+  GBA_E_ARG = -1,            /* invalid argument; nothing was changed */
+  GBA_E_ID_RANGE = -2,       /* a DIRECT id was outside [0, rows): the step was not applied */
+  GBA_E_OOM = -3,            /* device or pinned host allocation failed */
+  GBA_E_CUDA = -4,           /* a CUDA runtime call failed (see gba_last_error) */
+  GBA_E_DEVICE_TIMEOUT = -5, /* a bounded device-side wait gave up */
+  GBA_E_STATE = -6,          /* the handle failed earlier and accepts no more steps */
+  GBA_E_FULL = -7            /* the gradient buffer is full; apply, then push again */
+} gba_status;
+
+typedef enum { GBA_ADAGRAD = 0, GBA_ADAM = 1 } gba_optimizer;
+
+/* id -> row mapping of a table (no hash table on this path):
+ * DIRECT: the id is the row and must satisfy 0 <= id < rows;
+ * MODULO: row = (uint64_t)id % rows (hashing trick; colliding ids share a row). */
+typedef enum { GBA_ID_DIRECT = 0, GBA_ID_MODULO = 1 } gba_id_mode;
+
+/* Optimizer of a table or of the dense parameters.  Table 1 of the paper names
+ * Adagrad and Adam; the update rules are the textbook ones, one IEEE float
+ * operation at a time:
+ *   Adagrad: a += g*g;  w -= (lr*g) / sqrt(a)            (a starts at adagrad_init_acc > 0)
+ *   Adam:    m = b1*m + (1-b1)*g;  v = b2*v + (1-b2)*(g*g);
+ *            w -= (lr*(m/bc1)) / (sqrt(v/bc2) + eps),  bc_i = 1 - b_i^t, t = global step + 1 */
+typedef struct {
+  int32_t kind;            /* gba_optimizer */
+  float lr;
+  float adagrad_init_acc;  /* Adagrad only; paper default 0.1 */
+  float beta1, beta2, eps; /* Adam only; 0.9, 0.999, 1e-8 */
+} gba_opt_desc;
+
+/* One embedding table: rows x dim float32 weights plus optimizer state and a
+ * per-row step tag (Alg. 2 "global step of appearance tagged to each ID"). */
+typedef struct {
+  int64_t rows;            /* >= 1; the sum of rows over all tables must be < 2^32 */
+  int32_t dim;             /* 1 .. 256 */
+  int32_t id_mode;         /* gba_id_mode */
+  int64_t max_ids_per_msg; /* upper bound on one message's ids for this table (sizes the buffers) */
+  gba_opt_desc opt;
+} gba_table_desc;
+
+/* Staleness rule (Sec. 4.1 Eq. (1)): a gradient with staleness s is kept iff
+ * s <= iota; staleness = max(0, reference - token).
+ *   row_staleness 0: rows use the row's step tag as the reference (Alg. 2),
+ *                 1: rows use the current step k, like the dense gradient.
+ *   sparse_denominator 0: divide a row's kept sum by the number of messages in
+ *                 the global batch that contain the row (Alg. 2 "workers that
+ *                 encountered the particular ID"), 1: by the kept ones, 2: by M.
+ * iota = INT32_MAX keeps every gradient (BSP). */
+typedef struct {
+  int32_t iota;
+  int32_t row_staleness;
+  int32_t sparse_denominator;
+} gba_staleness_desc;
+
+/* The sparse part of one message for one table: n ids and n x dim gradient rows
+ * (row-major float32). */
+typedef struct {
+  const int64_t* ids;
+  int64_t n;
+  const float* rows;
+} gba_sparse_grad;
+
+/* Counters accumulated over all applied steps (Table 3 reports the number of
+ * excluded batches and the average / max staleness). */
+typedef struct {
+  int64_t steps;
+  int64_t msgs_kept, msgs_dropped;          /* dense decisions */
+  int64_t dense_stale_sum, dense_stale_max; /* over all popped messages */
+  int64_t pairs, pairs_dropped;             /* distinct (message, row) pairs */
+  int64_t row_stale_sum, row_stale_max;     /* over those pairs */
+  int64_t occurrences;                      /* id occurrences */
+  int64_t rows_touched, rows_applied;       /* unique rows; those that took a step */
+  int64_t occurrences_kept;                 /* occurrences whose gradient was aggregated */
+} gba_stats_t;
+
+/* Per kernel class: launches and device time summed since timing was enabled. */
+typedef struct {
+  int64_t launches[8];
+  double ms[8];
+} gba_kernel_times_t;
+/* indices into gba_kernel_times_t */
+enum {
+  GBA_K_WEIGHTS = 0, GBA_K_SORT_HIST = 1, GBA_K_SORT_PASS = 2, GBA_K_SEGSUM = 3,
+  GBA_K_FIXUP = 4, GBA_K_DENSE = 5, GBA_K_INIT = 6, GBA_K_OTHER = 7
+};
+
+/*
+ * gba_create - allocate the parameter-server state on the current device.
+ *
+ * tables[n_tables]   table descriptions (n_tables may be 0).
+ * dense_size         number of dense float32 parameters (may be 0).
+ * dense_opt          optimizer of the dense parameters (may be NULL if dense_size is 0).
+ * global_batch       G: a step is applied once the buffered local batches sum to >= G
+ *                    (Sec. 4.1: G_a = B_a * M equals the synchronous B_s * N_s).
+ * max_buffered_msgs  capacity of the gradient buffer, in messages (>= 1).
+ * st                 staleness rule (NULL: iota = INT32_MAX, tags, encountered).
+ * init_seed          weights are initialised from a counter-based hash of
+ *                    (seed, table, element); optimizer state from the descriptors.
+ * cuda_stream        cudaStream_t for all work of the handle; NULL makes a new one.
+ * out                receives the handle.
+ * Returns GBA_E_ARG for invalid descriptions, GBA_E_OOM / GBA_E_CUDA on failure.
+ */
+gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t dense_size,
+                      const gba_opt_desc* dense_opt, int64_t global_batch,
+                      int32_t max_buffered_msgs, const gba_staleness_desc* st,
+                      uint64_t init_seed, void* cuda_stream, gba_handle** out);
+
+/*
+ * gba_push - store one worker message in the gradient buffer (Alg. 2: "store
+ * the gradients with the token to the gradient buffer").
+ *
+ * token        the global step the worker's batch was issued at (>= 0; a
+ *              token ahead of the current step counts as staleness 0).
+ * per_table    n_tables entries; ids/rows may be device or host pointers
+ *              (host memory should be pinned for the copy to be asynchronous).
+ * dense_grad   dense_size floats, device or host.
+ * local_batch  the message's local batch size B (>= 1).
+ * The data are copied on the handle's stream; the caller may reuse its buffers
+ * once that copy is complete (stream order).  GBA_E_FULL when the buffer holds
+ * max_buffered_msgs messages; GBA_E_ARG for n > max_ids_per_msg or NULL data.
+ */
+gba_status gba_push(gba_handle* h, int64_t token, const gba_sparse_grad* per_table,
+                    const float* dense_grad, int32_t local_batch);
+
+/*
+ * gba_push_ref - like gba_push, but the library only records the pointers:
+ * the device buffers must stay valid and unmodified until the step that pops
+ * the message has completed on the stream.  Pointers must be device memory;
+ * dense_grad must be 16-byte aligned, and rows too when dim is a multiple of 4.
+ */
+gba_status gba_push_ref(gba_handle* h, int64_t token, const gba_sparse_grad* per_table,
+                        const float* dense_grad, int32_t local_batch);
+
+/*
+ * gba_try_apply - if the buffered local batches reach the global batch, pop the
+ * oldest messages that do (Alg. 2: "pop N_a gradients"), enqueue one global
+ * step on the stream and return 1; otherwise return 0.  The step:
+ *   Eq. (1) weights per message; rows deduplicated by id (radix sort);
+ *   per row: decay by the row's tag vs the token, sum of kept gradients divided
+ *   by the denominator, optimizer, tag := k + 1 (rows with no kept gradient are
+ *   left untouched); dense: sum of kept gradients / M, optimizer (always).
+ * A negative return is a gba_status (a latched device error surfaces here).
+ */
+int32_t gba_try_apply(gba_handle* h);
+
+/* gba_pull_version - the number of global steps applied so far (k); a worker
+ * that takes its token from here reports staleness k' - k when applied at k'. */
+int64_t gba_pull_version(gba_handle* h);
+
+/* gba_sync - wait for all work of the handle, then report any latched device error. */
+gba_status gba_sync(gba_handle* h);
+
+/* gba_get_table / gba_get_dense - device pointers to the state (borrowed, valid
+ * until gba_destroy): weights [rows*dim], slot0 (Adagrad accumulator or Adam m),
+ * slot1 (Adam v, NULL for Adagrad), per-row step tags [rows]. */
+gba_status gba_get_table(gba_handle* h, int32_t t, float** w, float** slot0, float** slot1,
+                         int32_t** ver);
+gba_status gba_get_dense(gba_handle* h, float** w, float** slot0, float** slot1);
+
+/* gba_stats - synchronise and copy the accumulated counters. */
+gba_status gba_stats(gba_handle* h, gba_stats_t* out);
+
+/* gba_last_error - text of the last failure of this handle ("" if none). */
+const char* gba_last_error(gba_handle* h);
+
+/* gba_destroy - wait for outstanding work and free everything (NULL is a no-op). */
+void gba_destroy(gba_handle* h);
+
+/* ---- instrumentation and test entry points ----------------------------- */
+
+/* gba_set_timing - when on, every kernel launch is bracketed by CUDA events on
+ * its stream; gba_kernel_times synchronises and returns the sums. */
+gba_status gba_set_timing(gba_handle* h, int32_t on);
+gba_status gba_kernel_times(gba_handle* h, gba_kernel_times_t* out);
+
+/* gba_set_debug - when on, each step also records the dedup result so that
+ * gba_debug_segments can return it (costs one extra write per unique row). */
+gba_status gba_set_debug(gba_handle* h, int32_t on);
+
+/*
+ * gba_debug_segments - dedup output of the last applied step (debug must have
+ * been on for it).  Host buffers of capacity cap receive, per unique row in
+ * increasing (table, row) order: table[i], row[i], count[i] (messages that
+ * contain the row) and kept[i] (kept occurrences).  *n_unique receives the
+ * number of unique rows (GBA_E_ARG if it exceeds cap).
+ */
+gba_status gba_debug_segments(gba_handle* h, int64_t cap, int32_t* table, int64_t* row,
+                              int64_t* count, int64_t* kept, int64_t* n_unique);
+
+/* gba_debug_sorted - the last step's sorted keys (global row = sum of the rows
+ * of earlier tables + row) and occurrence indices, into host buffers of
+ * capacity cap; *n receives the number of occurrences. */
+gba_status gba_debug_sorted(gba_handle* h, int64_t cap, uint32_t* keys, uint32_t* occ,
+                            int64_t* n);
+
+/* gba_debug_keep - message weights f (Eq. (1)) of the last step, in pop order. */
+gba_status gba_debug_keep(gba_handle* h, int32_t cap, int32_t* keep, int32_t* M);
+
+/* gba_debug_set_wait_limit - the time (ns) after which a device-side wait of
+ * this handle gives up and latches GBA_E_DEVICE_TIMEOUT (default 2e9). */
+gba_status gba_debug_set_wait_limit(gba_handle* h, int64_t ns);
+
+/*
+ * gba_selftest_wait_timeout - run the library's bounded device wait on a flag
+ * that nothing sets, with the given limit, on the given stream (NULL = default
+ * stream), and return the status the kernel reports: GBA_E_DEVICE_TIMEOUT when
+ * the wait gave up as designed.
+ */
+gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream);
+
+/* gba_version_string - library build identification. */
+const char* gba_version_string(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GBA_H_ */

@@ -1,0 +1,226 @@
+// K5 of the GBA aggregate-and-apply step: the dense parameters.
+//
+// g = (sum over kept messages m of grad_m) / M  (Alg. 2: weighted sum of the
+// dense gradients divided by N_a; Appendix A: v_k = (1/M) sum g), then Adagrad
+// or Adam in place -- one pass over HBM: every kept gradient is read once, the
+// weights and optimizer state are read and written once.
+//
+// Each persistent CTA walks tiles of 1024 parameters.  A producer warp streams
+// the tile's slice of every kept message into a ring of shared-memory stages
+// with 1-D bulk async copies (cp.async.bulk, completion counted on an mbarrier
+// per stage); eight consumer warps sum the slices with compensated float
+// arithmetic, release each stage on an "empty" mbarrier, and finish the tile
+// with the optimizer.  Every mbarrier wait is bounded in time; a wait that
+// gives up latches ERR_TIMEOUT, the CTA stops issuing copies, waits (bounded)
+// for the copies it already issued, and exits.
+#include "gba_internal.cuh"
+
+namespace gba {
+
+namespace {
+
+constexpr int DT = 1024;           // parameters per tile
+constexpr int STAGES = 16;         // 4 KB each
+constexpr int CONSUMER_WARPS = 8;  // 256 threads, one float4 each
+constexpr int DENSE_THREADS = (CONSUMER_WARPS + 1) * 32;
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0u;
+}
+
+// Bounded wait for the phase with the given parity; false if it gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if ((int64_t)(globaltimer_ns() - t0) > limit_ns) return false;
+  }
+  return true;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+__global__ void __launch_bounds__(DENSE_THREADS)
+    k_dense_apply(StepArgs a, DenseArgs da, StepScratch sc, ErrSink err, int64_t wait_ns) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  float* stage_buf = reinterpret_cast<float*>(smem_raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem_raw + (size_t)STAGES * DT * sizeof(float));
+  uint64_t* empty = full + STAGES;
+  __shared__ int s_abort;
+
+  if (*(volatile uint32_t*)err.dev & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid == 0) {
+    for (int i = 0; i < STAGES; ++i) {
+      mbar_init(full + i, 1u);
+      mbar_init(empty + i, (uint32_t)CONSUMER_WARPS);
+    }
+    s_abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+
+  const int n_kept = *sc.n_kept;
+  const int64_t D4 = da.D & ~3ll;  // parameters streamed by bulk copies
+  const int64_t n_tiles = (D4 + DT - 1) / DT;
+
+  if (warp == CONSUMER_WARPS) {
+    // ---- producer
+    if (lane == 0) {
+      uint32_t q = 0;
+      bool ok = true;
+      for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        const int64_t start = tile * DT;
+        const uint32_t bytes = (uint32_t)((D4 - start < DT ? D4 - start : DT) * sizeof(float));
+        for (int j = 0; j < n_kept; ++j, ++q) {
+          const int stage = (int)(q % STAGES);
+          const uint32_t ph = (q / STAGES) & 1u;
+          if (!mbar_wait(empty + stage, ph ^ 1u, wait_ns) || *(volatile int*)&s_abort) {
+            raise_error(err, ERR_TIMEOUT);
+            s_abort = 1;
+            ok = false;
+            break;
+          }
+          const float* src = a.dense_ptr[sc.kept_list[j]] + start;
+          mbar_arrive_expect_tx(full + stage, bytes);
+          bulk_g2s(stage_buf + (size_t)stage * DT, src, bytes, full + stage);
+        }
+      }
+      // Make sure no copy this CTA issued is still landing when it exits.  The
+      // copies read valid memory and land within microseconds; this wait has its
+      // own one-second bound, independent of the configurable limit.
+      const uint32_t n_drain = q < (uint32_t)STAGES ? q : (uint32_t)STAGES;
+      for (uint32_t i = 0; i < n_drain; ++i) {
+        const uint32_t qq = q - 1 - i;
+        mbar_wait(full + (qq % STAGES), (qq / STAGES) & 1u, 1000000000ll);
+      }
+    }
+  } else {
+    // ---- consumers: thread c owns parameters [4c, 4c + 4) of each tile
+    const int c = tid;
+    const float Mf = (float)da.M;
+    uint32_t q = 0;
+    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+      const int64_t start = tile * DT;
+      const int64_t n = D4 - start < DT ? D4 - start : DT;
+      const bool mine = (int64_t)c * 4 < n;
+      const int64_t e = start + (int64_t)c * 4;
+      float4 w = make_float4(0.f, 0.f, 0.f, 0.f), s0 = w, s1 = w;
+      if (mine) {
+        w = *reinterpret_cast<const float4*>(da.w + e);
+        s0 = *reinterpret_cast<const float4*>(da.s0 + e);
+        if (da.opt.kind == 1) s1 = *reinterpret_cast<const float4*>(da.s1 + e);
+      }
+      CSum acc[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[i] = CSum{0.f, 0.f};
+      bool aborted = false;
+      for (int j = 0; j < n_kept; ++j, ++q) {
+        const int stage = (int)(q % STAGES);
+        const uint32_t ph = (q / STAGES) & 1u;
+        // Every lane waits (acquiring the copied bytes); the verdict is made
+        // warp-uniform so the warp leaves the loop together.
+        bool ok = mbar_wait(full + stage, ph, wait_ns);
+        ok = __all_sync(0xffffffffu, ok) &&
+             __shfl_sync(0xffffffffu, *(volatile int*)&s_abort, 0) == 0;
+        if (!ok) {
+          if (lane == 0) {
+            raise_error(err, ERR_TIMEOUT);
+            s_abort = 1;
+          }
+          aborted = true;
+          break;
+        }
+        if (mine) {
+          const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT + 4 * c);
+          csum_add(acc[0], v.x);
+          csum_add(acc[1], v.y);
+          csum_add(acc[2], v.z);
+          csum_add(acc[3], v.w);
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty + stage);
+      }
+      if (aborted) break;
+      if (mine) {
+        float wv[4] = {w.x, w.y, w.z, w.w}, a0[4] = {s0.x, s0.y, s0.z, s0.w},
+              a1[4] = {s1.x, s1.y, s1.z, s1.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) opt_update(da.opt, wv[i], a0[i], a1[i],
+                                               __fdiv_rn(csum_value(acc[i]), Mf));
+        *reinterpret_cast<float4*>(da.w + e) = make_float4(wv[0], wv[1], wv[2], wv[3]);
+        *reinterpret_cast<float4*>(da.s0 + e) = make_float4(a0[0], a0[1], a0[2], a0[3]);
+        if (da.opt.kind == 1)
+          *reinterpret_cast<float4*>(da.s1 + e) = make_float4(a1[0], a1[1], a1[2], a1[3]);
+      }
+    }
+    // The last (D mod 4) parameters: plain loads, CTA 0.
+    if (blockIdx.x == 0 && c < (int)(da.D - D4)) {
+      const int64_t e = D4 + c;
+      CSum acc{0.f, 0.f};
+      for (int j = 0; j < n_kept; ++j) csum_add(acc, a.dense_ptr[sc.kept_list[j]][e]);
+      float wv = da.w[e], a0 = da.s0[e], a1 = da.opt.kind == 1 ? da.s1[e] : 0.f;
+      opt_update(da.opt, wv, a0, a1, __fdiv_rn(csum_value(acc), Mf));
+      da.w[e] = wv;
+      da.s0[e] = a0;
+      if (da.opt.kind == 1) da.s1[e] = a1;
+    }
+  }
+  __syncthreads();
+}
+
+}  // namespace
+
+size_t dense_smem_bytes() { return (size_t)STAGES * DT * sizeof(float) + 2 * STAGES * sizeof(uint64_t); }
+
+cudaError_t configure_dense() {
+  return cudaFuncSetAttribute(k_dense_apply, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)dense_smem_bytes());
+}
+
+void launch_dense(const StepArgs& a, const DenseArgs& da, StepScratch sc, ErrSink err,
+                  int64_t wait_ns, int num_sms, cudaStream_t s) {
+  const size_t smem = dense_smem_bytes();
+  const int64_t n_tiles = ((da.D & ~3ll) + DT - 1) / DT;
+  int64_t grid = (int64_t)num_sms * 3;
+  if (grid > n_tiles) grid = n_tiles;
+  if (grid < 1) grid = 1;
+  k_dense_apply<<<(unsigned)grid, DENSE_THREADS, smem, s>>>(a, da, sc, err, wait_ns);
+}
+
+}  // namespace gba

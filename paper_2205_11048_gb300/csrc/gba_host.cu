@@ -1,0 +1,1010 @@
+// Host side of libgba: the gradient buffer (FIFO of messages and the device
+// buffers their data live in), the assembly of a global step, kernel launches
+// on the handle's stream, error latching and the C ABI of include/gba.h.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <deque>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "gba.h"
+#include "gba_internal.cuh"
+
+using namespace gba;
+
+namespace {
+
+constexpr int MAX_DIM = 256;
+constexpr int META_SLOTS = 4;
+constexpr int MAX_PASSES = 4;
+constexpr int64_t MAX_STEP_OCC = (1ll << 30) - 1;
+
+struct Arena {  // contiguous-allocation ring over [0, cap) with virtual offsets
+  int64_t cap = 0;
+  int64_t vhead = 0, vtail = 0;
+  int64_t* ids = nullptr;
+  float* rows = nullptr;
+
+  int64_t alloc(int64_t n) {
+    if (n == 0) return vtail;
+    int64_t v = vtail;
+    if ((v % cap) + n > cap) v = (v / cap + 1) * cap;  // do not wrap inside a message
+    if (v + n - vhead > cap) return -1;
+    vtail = v + n;
+    return v;
+  }
+  void release_through(int64_t v_end) { vhead = std::max(vhead, v_end); }
+};
+
+struct TableState {
+  gba_table_desc desc;
+  float* w = nullptr;
+  float* s0 = nullptr;
+  float* s1 = nullptr;
+  int32_t* ver = nullptr;
+  uint32_t key_base = 0;
+  double bpow1 = 1.0, bpow2 = 1.0;  // beta^t of Adam, as successive products
+  Arena arena;
+};
+
+struct Msg {
+  int64_t token;
+  int32_t B;
+  bool copied;
+  const float* dense;
+  std::vector<const int64_t*> ids;
+  std::vector<const float*> rows;
+  std::vector<int64_t> n;
+  std::vector<int64_t> arena_v;  // virtual start in each table's arena (copied messages)
+};
+
+struct PendingTiming {
+  int kind;
+  cudaEvent_t a, b;
+};
+
+size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
+
+}  // namespace
+
+struct gba_handle {
+  int device = 0;
+  int num_sms = 152;
+  cudaStream_t stream = nullptr;
+  bool own_stream = false;
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+
+  std::vector<TableState> tables;
+  int32_t T = 0;
+  int64_t D = 0;
+  int64_t D_pad = 0;
+  gba_opt_desc dense_opt{};
+  float* dw = nullptr;
+  float* ds0 = nullptr;
+  float* ds1 = nullptr;
+  double dbpow1 = 1.0, dbpow2 = 1.0;
+  int64_t G = 1;
+  int32_t max_buf = 1;
+  gba_staleness_desc st{};
+  uint64_t seed = 0;
+  int64_t k = 0;
+  uint32_t total_keys_bits = 1;
+  int passes = 1;
+
+  std::deque<Msg> fifo;
+  bool arenas_ready = false;
+  float* dense_ring = nullptr;
+  int32_t slot_head = 0, slot_count = 0;
+
+  TableInfo* d_tinfo = nullptr;
+  std::vector<TableInfo> h_tinfo;
+
+  size_t meta_bytes = 0;
+  char* d_meta = nullptr;
+  char* h_meta[META_SLOTS] = {};
+  cudaEvent_t meta_ev[META_SLOTS] = {};
+  int meta_slot = 0;
+
+  // sort / segment scratch, grown on demand
+  int64_t n_cap = 0;
+  uint32_t* d_keys[2] = {};
+  uint32_t* d_vals[2] = {};
+  unsigned long long* d_status = nullptr;
+  int64_t status_tiles = 0;
+  uint32_t epoch = 0;
+  uint32_t* d_dbg_count = nullptr;
+  uint32_t* d_dbg_kept = nullptr;
+  int64_t dbg_cap = 0;
+  char* d_step_scratch = nullptr;
+  StepScratch sc{};
+  SegRecords rec{};
+  int64_t rec_warps = 0;
+  int d_max = 1;
+
+  uint32_t* d_err = nullptr;
+  uint32_t* h_err = nullptr;  // mapped pinned
+  ErrSink sink{};
+  DevStats* d_stats = nullptr;
+  bool failed = false;
+  gba_status fail_code = GBA_OK;
+  std::string last_error;
+  int64_t wait_ns = 2000000000ll;
+
+  bool debug = false;
+  bool timing = false;
+  std::vector<PendingTiming> pending;
+  std::vector<cudaEvent_t> event_pool;
+  gba_kernel_times_t times{};
+
+  // last applied step, for the debug entry points
+  bool have_last = false;
+  int64_t last_N = 0;
+  int last_buf = 0;
+  int32_t last_M = 0;
+};
+
+namespace {
+
+gba_status set_err(gba_handle* h, gba_status s, const std::string& msg) {
+  if (h) h->last_error = msg;
+  return s;
+}
+
+gba_status cuda_fail(gba_handle* h, cudaError_t e, const char* what) {
+  std::string m = std::string(what) + ": " + cudaGetErrorString(e);
+  if (h) h->last_error = m;
+  return e == cudaErrorMemoryAllocation ? GBA_E_OOM : GBA_E_CUDA;
+}
+
+#define GBA_CUDA(h, call)                                    \
+  do {                                                       \
+    cudaError_t e_ = (call);                                 \
+    if (e_ != cudaSuccess) return cuda_fail((h), e_, #call); \
+  } while (0)
+
+cudaEvent_t take_event(gba_handle* h) {
+  if (!h->event_pool.empty()) {
+    cudaEvent_t e = h->event_pool.back();
+    h->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Brackets one launch with events when timing is on; always counts launches.
+struct Timed {
+  gba_handle* h;
+  int kind;
+  cudaStream_t s;
+  cudaEvent_t a = nullptr;
+  Timed(gba_handle* h_, int kind_, cudaStream_t s_) : h(h_), kind(kind_), s(s_) {
+    h->times.launches[kind]++;
+    if (h->timing) {
+      a = take_event(h);
+      cudaEventRecord(a, s);
+    }
+  }
+  ~Timed() {
+    if (h->timing) {
+      cudaEvent_t b = take_event(h);
+      cudaEventRecord(b, s);
+      h->pending.push_back({kind, a, b});
+    }
+  }
+};
+
+void collect_timing(gba_handle* h) {
+  for (auto& p : h->pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, p.a, p.b) == cudaSuccess) h->times.ms[p.kind] += ms;
+    h->event_pool.push_back(p.a);
+    h->event_pool.push_back(p.b);
+  }
+  h->pending.clear();
+}
+
+gba_status validate_opt(const gba_opt_desc& o) {
+  if (o.kind != GBA_ADAGRAD && o.kind != GBA_ADAM) return GBA_E_ARG;
+  if (!std::isfinite(o.lr)) return GBA_E_ARG;
+  if (o.kind == GBA_ADAGRAD && !(o.adagrad_init_acc > 0.f && std::isfinite(o.adagrad_init_acc)))
+    return GBA_E_ARG;
+  if (o.kind == GBA_ADAM && !(o.beta1 >= 0.f && o.beta1 < 1.f && o.beta2 >= 0.f &&
+                              o.beta2 < 1.f && o.eps >= 0.f && std::isfinite(o.eps)))
+    return GBA_E_ARG;
+  return GBA_OK;
+}
+
+// Adam bias corrections and constants for the next step of one parameter group.
+OptStep make_opt_step(const gba_opt_desc& o, double bpow1_next, double bpow2_next) {
+  OptStep s{};
+  s.kind = o.kind;
+  s.lr = o.lr;
+  s.b1 = o.beta1;
+  s.b2 = o.beta2;
+  s.eps = o.eps;
+  s.c1 = 1.0f - o.beta1;
+  s.c2 = 1.0f - o.beta2;
+  s.bc1 = (float)(1.0 - bpow1_next);
+  s.bc2 = (float)(1.0 - bpow2_next);
+  return s;
+}
+
+void free_all(gba_handle* h) {
+  if (!h) return;
+  cudaSetDevice(h->device);
+  if (h->stream) cudaStreamSynchronize(h->stream);
+  if (h->side) cudaStreamSynchronize(h->side);
+  for (auto& t : h->tables) {
+    cudaFree(t.w);
+    cudaFree(t.s0);
+    cudaFree(t.s1);
+    cudaFree(t.ver);
+    cudaFree(t.arena.ids);
+    cudaFree(t.arena.rows);
+  }
+  cudaFree(h->dw);
+  cudaFree(h->ds0);
+  cudaFree(h->ds1);
+  cudaFree(h->dense_ring);
+  cudaFree(h->d_tinfo);
+  cudaFree(h->d_meta);
+  for (int i = 0; i < META_SLOTS; ++i) {
+    if (h->h_meta[i]) cudaFreeHost(h->h_meta[i]);
+    if (h->meta_ev[i]) cudaEventDestroy(h->meta_ev[i]);
+  }
+  for (int i = 0; i < 2; ++i) {
+    cudaFree(h->d_keys[i]);
+    cudaFree(h->d_vals[i]);
+  }
+  cudaFree(h->d_status);
+  cudaFree(h->d_dbg_count);
+  cudaFree(h->d_dbg_kept);
+  cudaFree(h->d_step_scratch);
+  cudaFree(h->rec.hi);
+  cudaFree(h->rec.lo);
+  cudaFree(h->rec.meta);
+  cudaFree(h->d_err);
+  if (h->h_err) cudaFreeHost(h->h_err);
+  cudaFree(h->d_stats);
+  for (auto& p : h->pending) {
+    cudaEventDestroy(p.a);
+    cudaEventDestroy(p.b);
+  }
+  for (auto e : h->event_pool) cudaEventDestroy(e);
+  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
+  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->side) cudaStreamDestroy(h->side);
+  if (h->own_stream && h->stream) cudaStreamDestroy(h->stream);
+}
+
+// Device error latched by a kernel?  Polls the mapped flag without
+// synchronising; if set, synchronises and turns the word into a status.
+gba_status poll_device_error(gba_handle* h, bool force_sync) {
+  if (!force_sync && *(volatile uint32_t*)h->h_err == 0u) return GBA_OK;
+  cudaStreamSynchronize(h->side);
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e != cudaSuccess) {
+    h->failed = true;
+    h->fail_code = cuda_fail(h, e, "stream synchronize");
+    return h->fail_code;
+  }
+  uint32_t word = 0;
+  e = cudaMemcpy(&word, h->d_err, sizeof word, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) {
+    h->failed = true;
+    h->fail_code = cuda_fail(h, e, "read device error word");
+    return h->fail_code;
+  }
+  if (word == 0u) return GBA_OK;
+  h->failed = true;
+  if (word & ERR_ID_RANGE) {
+    h->fail_code = set_err(h, GBA_E_ID_RANGE, "an id outside [0, rows) in a DIRECT table");
+  } else if (word & ERR_TIMEOUT) {
+    h->fail_code = set_err(h, GBA_E_DEVICE_TIMEOUT, "a bounded device wait gave up");
+  } else {
+    h->fail_code = set_err(h, GBA_E_CUDA, "device consistency check failed");
+  }
+  return h->fail_code;
+}
+
+gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
+  if (N > h->n_cap) {
+    cudaStreamSynchronize(h->side);
+    cudaStreamSynchronize(h->stream);
+    int64_t cap = std::max<int64_t>(N + N / 4, 4096);
+    for (int i = 0; i < 2; ++i) {
+      cudaFree(h->d_keys[i]);
+      cudaFree(h->d_vals[i]);
+      h->d_keys[i] = h->d_vals[i] = nullptr;
+      GBA_CUDA(h, cudaMalloc(&h->d_keys[i], cap * sizeof(uint32_t)));
+      GBA_CUDA(h, cudaMalloc(&h->d_vals[i], cap * sizeof(uint32_t)));
+    }
+    h->n_cap = cap;
+    const int64_t tiles = sort_tiles(cap);
+    cudaFree(h->d_status);
+    h->d_status = nullptr;
+    GBA_CUDA(h, cudaMalloc(&h->d_status, (size_t)tiles * 256 * sizeof(unsigned long long)));
+    GBA_CUDA(h, cudaMemset(h->d_status, 0, (size_t)tiles * 256 * sizeof(unsigned long long)));
+    h->status_tiles = tiles;
+  }
+  if (h->debug && N > h->dbg_cap) {
+    cudaStreamSynchronize(h->stream);
+    cudaFree(h->d_dbg_count);
+    cudaFree(h->d_dbg_kept);
+    h->d_dbg_count = h->d_dbg_kept = nullptr;
+    const int64_t cap = std::max<int64_t>(h->n_cap, N);
+    GBA_CUDA(h, cudaMalloc(&h->d_dbg_count, cap * sizeof(uint32_t)));
+    GBA_CUDA(h, cudaMalloc(&h->d_dbg_kept, cap * sizeof(uint32_t)));
+    h->dbg_cap = cap;
+  }
+  return GBA_OK;
+}
+
+gba_status ensure_arenas(gba_handle* h) {
+  if (h->arenas_ready) return GBA_OK;
+  for (auto& t : h->tables) {
+    const int64_t cap = (int64_t)(h->max_buf + 1) * std::max<int64_t>(1, t.desc.max_ids_per_msg);
+    t.arena.cap = cap;
+    GBA_CUDA(h, cudaMalloc(&t.arena.ids, cap * sizeof(int64_t)));
+    GBA_CUDA(h, cudaMalloc(&t.arena.rows, cap * (size_t)t.desc.dim * sizeof(float)));
+  }
+  if (h->D > 0) {
+    const size_t bytes = (size_t)h->max_buf * h->D_pad * sizeof(float);
+    GBA_CUDA(h, cudaMalloc(&h->dense_ring, bytes));
+    GBA_CUDA(h, cudaMemset(h->dense_ring, 0, bytes));
+  }
+  h->arenas_ready = true;
+  return GBA_OK;
+}
+
+gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_table,
+                       const float* dense_grad, int32_t local_batch, bool copy) {
+  if (!h) return GBA_E_ARG;
+  if (h->failed) return set_err(h, GBA_E_STATE, "handle failed earlier");
+  if (token < 0) return set_err(h, GBA_E_ARG, "token < 0");
+  if (local_batch < 1) return set_err(h, GBA_E_ARG, "local_batch < 1");
+  if (h->T > 0 && !per_table) return set_err(h, GBA_E_ARG, "per_table is NULL");
+  if (h->D > 0 && !dense_grad) return set_err(h, GBA_E_ARG, "dense_grad is NULL");
+  for (int t = 0; t < h->T; ++t) {
+    const gba_sparse_grad& g = per_table[t];
+    const gba_table_desc& d = h->tables[t].desc;
+    if (g.n < 0 || g.n > d.max_ids_per_msg)
+      return set_err(h, GBA_E_ARG, "ids per message outside [0, max_ids_per_msg]");
+    if (g.n > 0 && (!g.ids || !g.rows)) return set_err(h, GBA_E_ARG, "NULL ids or rows");
+    if (!copy && g.n > 0) {
+      if (((uintptr_t)g.ids & 7u) != 0) return set_err(h, GBA_E_ARG, "ids not 8-byte aligned");
+      if (d.dim % 4 == 0 && ((uintptr_t)g.rows & 15u) != 0)
+        return set_err(h, GBA_E_ARG, "rows not 16-byte aligned");
+      if (((uintptr_t)g.rows & 3u) != 0) return set_err(h, GBA_E_ARG, "rows not 4-byte aligned");
+    }
+  }
+  if (!copy && h->D > 0 && ((uintptr_t)dense_grad & 15u) != 0)
+    return set_err(h, GBA_E_ARG, "dense_grad not 16-byte aligned");
+  if ((int64_t)h->fifo.size() >= h->max_buf) return set_err(h, GBA_E_FULL, "gradient buffer full");
+
+  Msg m;
+  m.token = token;
+  m.B = local_batch;
+  m.copied = copy;
+  m.ids.resize(h->T);
+  m.rows.resize(h->T);
+  m.n.resize(h->T);
+  m.arena_v.assign(h->T, -1);
+  if (copy) {
+    gba_status s = ensure_arenas(h);
+    if (s != GBA_OK) return s;
+    if (h->D > 0 && h->slot_count >= h->max_buf)
+      return set_err(h, GBA_E_FULL, "gradient buffer full");
+    std::vector<int64_t> saved_tail(h->T);
+    for (int t = 0; t < h->T; ++t) saved_tail[t] = h->tables[t].arena.vtail;
+    for (int t = 0; t < h->T; ++t) {
+      const int64_t n = per_table[t].n;
+      const int64_t v = h->tables[t].arena.alloc(n);
+      if (v < 0) {
+        for (int u = 0; u < h->T; ++u) h->tables[u].arena.vtail = saved_tail[u];
+        return set_err(h, GBA_E_FULL, "gradient buffer full (id storage)");
+      }
+      m.arena_v[t] = v;
+    }
+    for (int t = 0; t < h->T; ++t) {
+      const int64_t n = per_table[t].n;
+      Arena& ar = h->tables[t].arena;
+      const int64_t p = m.arena_v[t] % ar.cap;
+      const int32_t dim = h->tables[t].desc.dim;
+      m.ids[t] = ar.ids + p;
+      m.rows[t] = ar.rows + p * dim;
+      m.n[t] = n;
+      if (n > 0) {
+        GBA_CUDA(h, cudaMemcpyAsync(ar.ids + p, per_table[t].ids, n * sizeof(int64_t),
+                                    cudaMemcpyDefault, h->stream));
+        GBA_CUDA(h, cudaMemcpyAsync(ar.rows + p * dim, per_table[t].rows,
+                                    n * dim * sizeof(float), cudaMemcpyDefault, h->stream));
+      }
+    }
+    if (h->D > 0) {
+      const int32_t slot = (h->slot_head + h->slot_count) % h->max_buf;
+      float* dst = h->dense_ring + (size_t)slot * h->D_pad;
+      GBA_CUDA(h, cudaMemcpyAsync(dst, dense_grad, h->D * sizeof(float), cudaMemcpyDefault,
+                                  h->stream));
+      h->slot_count++;
+      m.dense = dst;
+    } else {
+      m.dense = nullptr;
+    }
+  } else {
+    for (int t = 0; t < h->T; ++t) {
+      m.ids[t] = per_table[t].ids;
+      m.rows[t] = per_table[t].rows;
+      m.n[t] = per_table[t].n;
+    }
+    m.dense = dense_grad;
+  }
+  h->fifo.push_back(std::move(m));
+  return GBA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t dense_size,
+                      const gba_opt_desc* dense_opt, int64_t global_batch,
+                      int32_t max_buffered_msgs, const gba_staleness_desc* st,
+                      uint64_t init_seed, void* cuda_stream, gba_handle** out) {
+  if (!out) return GBA_E_ARG;
+  *out = nullptr;
+  if (n_tables < 0 || (n_tables > 0 && !tables)) return GBA_E_ARG;
+  if (dense_size < 0 || (dense_size > 0 && !dense_opt)) return GBA_E_ARG;
+  if (global_batch < 1 || max_buffered_msgs < 1) return GBA_E_ARG;
+  uint64_t total_rows = 0;
+  for (int t = 0; t < n_tables; ++t) {
+    const gba_table_desc& d = tables[t];
+    if (d.rows < 1 || d.dim < 1 || d.dim > MAX_DIM) return GBA_E_ARG;
+    if (d.id_mode != GBA_ID_DIRECT && d.id_mode != GBA_ID_MODULO) return GBA_E_ARG;
+    if (d.max_ids_per_msg < 0 || d.max_ids_per_msg > MAX_STEP_OCC) return GBA_E_ARG;
+    if (validate_opt(d.opt) != GBA_OK) return GBA_E_ARG;
+    total_rows += (uint64_t)d.rows;
+  }
+  if (total_rows >= 0xFFFFFFFFull) return GBA_E_ARG;  // keys are 32-bit, one value reserved
+  if (dense_size > 0 && validate_opt(*dense_opt) != GBA_OK) return GBA_E_ARG;
+  gba_staleness_desc rule{0x7FFFFFFF, 0, 0};
+  if (st) rule = *st;
+  if (rule.iota < 0 || (rule.row_staleness != 0 && rule.row_staleness != 1) ||
+      rule.sparse_denominator < 0 || rule.sparse_denominator > 2)
+    return GBA_E_ARG;
+
+  gba_handle* h = new (std::nothrow) gba_handle();
+  if (!h) return GBA_E_OOM;
+  h->T = n_tables;
+  h->D = dense_size;
+  h->D_pad = (dense_size + 3) & ~3ll;
+  if (dense_opt) h->dense_opt = *dense_opt;
+  h->G = global_batch;
+  h->max_buf = max_buffered_msgs;
+  h->st = rule;
+  h->seed = init_seed;
+
+  auto fail = [&](gba_status s) {
+    free_all(h);
+    delete h;
+    return s;
+  };
+  cudaError_t e = cudaGetDevice(&h->device);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return fail(GBA_E_CUDA);
+  }
+  int sms = 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, h->device) == cudaSuccess &&
+      sms > 0)
+    h->num_sms = sms;
+  if (cuda_stream) {
+    h->stream = (cudaStream_t)cuda_stream;
+  } else {
+    if (cudaStreamCreateWithFlags(&h->stream, cudaStreamNonBlocking) != cudaSuccess)
+      return fail(GBA_E_CUDA);
+    h->own_stream = true;
+  }
+  if (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess)
+    return fail(GBA_E_CUDA);
+  if (configure_dense() != cudaSuccess) return fail(GBA_E_CUDA);
+
+  // key space: tables in order
+  uint32_t base = 0;
+  h->tables.resize(n_tables);
+  h->h_tinfo.resize(n_tables);
+  for (int t = 0; t < n_tables; ++t) {
+    TableState& ts = h->tables[t];
+    ts.desc = tables[t];
+    ts.key_base = base;
+    h->h_tinfo[t] = TableInfo{tables[t].rows, base, tables[t].id_mode};
+    base += (uint32_t)tables[t].rows;
+    h->d_max = std::max(h->d_max, (int)tables[t].dim);
+  }
+  {
+    uint64_t kmax = total_rows > 0 ? total_rows - 1 : 0;
+    uint32_t bits = 1;
+    while (bits < 32 && (kmax >> bits) != 0) ++bits;
+    h->total_keys_bits = bits;
+    h->passes = (int)((bits + 7) / 8);
+  }
+
+  auto dev_alloc = [&](void** p, size_t bytes) -> bool {
+    if (bytes == 0) return true;
+    return cudaMalloc(p, bytes) == cudaSuccess;
+  };
+  for (int t = 0; t < n_tables; ++t) {
+    TableState& ts = h->tables[t];
+    const size_t n = (size_t)ts.desc.rows * ts.desc.dim;
+    if (!dev_alloc((void**)&ts.w, n * 4) || !dev_alloc((void**)&ts.s0, n * 4) ||
+        (ts.desc.opt.kind == GBA_ADAM && !dev_alloc((void**)&ts.s1, n * 4)) ||
+        !dev_alloc((void**)&ts.ver, (size_t)ts.desc.rows * 4))
+      return fail(GBA_E_OOM);
+  }
+  if (h->D > 0) {
+    if (!dev_alloc((void**)&h->dw, h->D_pad * 4) || !dev_alloc((void**)&h->ds0, h->D_pad * 4) ||
+        (h->dense_opt.kind == GBA_ADAM && !dev_alloc((void**)&h->ds1, h->D_pad * 4)))
+      return fail(GBA_E_OOM);
+  }
+  if (n_tables > 0) {
+    if (!dev_alloc((void**)&h->d_tinfo, n_tables * sizeof(TableInfo))) return fail(GBA_E_OOM);
+    if (cudaMemcpy(h->d_tinfo, h->h_tinfo.data(), n_tables * sizeof(TableInfo),
+                   cudaMemcpyHostToDevice) != cudaSuccess)
+      return fail(GBA_E_CUDA);
+  }
+  // step descriptor buffers
+  {
+    const size_t M = (size_t)max_buffered_msgs, T = (size_t)n_tables;
+    h->meta_bytes = align16(M * 8) + align16(M * 8) + align16(T * (M + 1) * 4) +
+                    align16(T * M * 8) + align16(T * M * 8) + align16((T + 1) * 8);
+    if (!dev_alloc((void**)&h->d_meta, h->meta_bytes)) return fail(GBA_E_OOM);
+    for (int i = 0; i < META_SLOTS; ++i) {
+      if (cudaHostAlloc((void**)&h->h_meta[i], h->meta_bytes, cudaHostAllocDefault) !=
+              cudaSuccess ||
+          cudaEventCreateWithFlags(&h->meta_ev[i], cudaEventDisableTiming) != cudaSuccess)
+        return fail(GBA_E_OOM);
+    }
+  }
+  {
+    const size_t M = (size_t)max_buffered_msgs;
+    const size_t bytes = align16(MAX_PASSES * 256 * 4) + align16(MAX_PASSES * 4) +
+                         align16(M * 4) + align16(M * 4) + align16(4);
+    if (!dev_alloc((void**)&h->d_step_scratch, bytes)) return fail(GBA_E_OOM);
+    char* p = h->d_step_scratch;
+    h->sc.hist = (uint32_t*)p;
+    p += align16(MAX_PASSES * 256 * 4);
+    h->sc.tile_counter = (uint32_t*)p;
+    p += align16(MAX_PASSES * 4);
+    h->sc.keep = (int32_t*)p;
+    p += align16(M * 4);
+    h->sc.kept_list = (int32_t*)p;
+    p += align16(M * 4);
+    h->sc.n_kept = (int32_t*)p;
+  }
+  {
+    h->rec_warps = (int64_t)h->num_sms * 32 + 64;
+    const size_t nf = (size_t)h->rec_warps * 2 * h->d_max;
+    if (!dev_alloc((void**)&h->rec.hi, nf * 4) || !dev_alloc((void**)&h->rec.lo, nf * 4) ||
+        !dev_alloc((void**)&h->rec.meta, (size_t)h->rec_warps * 2 * 6 * 4))
+      return fail(GBA_E_OOM);
+  }
+  if (!dev_alloc((void**)&h->d_err, 4) || !dev_alloc((void**)&h->d_stats, sizeof(DevStats)))
+    return fail(GBA_E_OOM);
+  if (cudaHostAlloc((void**)&h->h_err, 4, cudaHostAllocMapped) != cudaSuccess)
+    return fail(GBA_E_OOM);
+  *h->h_err = 0u;
+  uint32_t* h_err_dev = nullptr;
+  if (cudaHostGetDevicePointer((void**)&h_err_dev, h->h_err, 0) != cudaSuccess)
+    return fail(GBA_E_CUDA);
+  h->sink = ErrSink{h->d_err, h_err_dev};
+  if (cudaMemsetAsync(h->d_err, 0, 4, h->stream) != cudaSuccess ||
+      cudaMemsetAsync(h->d_stats, 0, sizeof(DevStats), h->stream) != cudaSuccess)
+    return fail(GBA_E_CUDA);
+
+  // initial values (R11 of the design notes: counter-based hash of (seed, array, element))
+  for (int t = 0; t < n_tables; ++t) {
+    TableState& ts = h->tables[t];
+    Timed tm(h, GBA_K_INIT, h->stream);
+    launch_init_table(ts.w, ts.s0, ts.s1, ts.ver, ts.desc.rows, ts.desc.dim, ts.desc.opt.kind,
+                      ts.desc.opt.adagrad_init_acc, init_seed, ((uint64_t)(uint32_t)t + 1u) << 48,
+                      h->stream);
+  }
+  if (h->D > 0) {
+    Timed tm(h, GBA_K_INIT, h->stream);
+    launch_init_dense(h->dw, h->ds0, h->ds1, h->D, h->dense_opt.kind,
+                      h->dense_opt.adagrad_init_acc, init_seed, (uint64_t)0xFFFFu << 48,
+                      h->stream);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(GBA_E_CUDA);
+  if (cudaStreamSynchronize(h->stream) != cudaSuccess) return fail(GBA_E_CUDA);
+  collect_timing(h);
+  *out = h;
+  return GBA_OK;
+}
+
+gba_status gba_push(gba_handle* h, int64_t token, const gba_sparse_grad* per_table,
+                    const float* dense_grad, int32_t local_batch) {
+  return push_common(h, token, per_table, dense_grad, local_batch, true);
+}
+
+gba_status gba_push_ref(gba_handle* h, int64_t token, const gba_sparse_grad* per_table,
+                        const float* dense_grad, int32_t local_batch) {
+  return push_common(h, token, per_table, dense_grad, local_batch, false);
+}
+
+int32_t gba_try_apply(gba_handle* h) {
+  if (!h) return GBA_E_ARG;
+  if (h->failed) return GBA_E_STATE;
+  {
+    gba_status s = poll_device_error(h, false);
+    if (s != GBA_OK) return s;
+  }
+  // Alg. 2: apply once the buffered local batches reach the global batch.
+  int64_t acc = 0;
+  int32_t M = 0;
+  for (const Msg& m : h->fifo) {
+    acc += m.B;
+    ++M;
+    if (acc >= h->G) break;
+  }
+  if (acc < h->G) return 0;
+  const int T = h->T;
+  std::vector<int64_t> nbase(T + 1, 0);
+  for (int t = 0; t < T; ++t) {
+    int64_t nt = 0;
+    for (int i = 0; i < M; ++i) nt += h->fifo[i].n[t];
+    nbase[t + 1] = nbase[t] + nt;
+  }
+  const int64_t N = nbase[T];
+  if (N > MAX_STEP_OCC) return set_err(h, GBA_E_ARG, "more than 2^30-1 ids in one global step");
+  cudaSetDevice(h->device);
+  {
+    gba_status s = ensure_step_capacity(h, N);
+    if (s != GBA_OK) return s;
+  }
+
+  // ---- step descriptor
+  const int slot = h->meta_slot;
+  h->meta_slot = (h->meta_slot + 1) % META_SLOTS;
+  cudaEventSynchronize(h->meta_ev[slot]);
+  char* hp = h->h_meta[slot];
+  const size_t Mx = (size_t)h->max_buf;
+  size_t off = 0;
+  auto section = [&](size_t bytes) {
+    size_t o = off;
+    off += align16(bytes);
+    return o;
+  };
+  const size_t o_tok = section(Mx * 8), o_dense = section(Mx * 8),
+               o_off = section((size_t)T * (Mx + 1) * 4), o_ids = section((size_t)T * Mx * 8),
+               o_rows = section((size_t)T * Mx * 8), o_nbase = section((size_t)(T + 1) * 8);
+  int64_t* tok = (int64_t*)(hp + o_tok);
+  const float** dptr = (const float**)(hp + o_dense);
+  uint32_t* moff = (uint32_t*)(hp + o_off);
+  const int64_t** iptr = (const int64_t**)(hp + o_ids);
+  const float** rptr = (const float**)(hp + o_rows);
+  int64_t* nb = (int64_t*)(hp + o_nbase);
+  for (int i = 0; i < M; ++i) {
+    const Msg& m = h->fifo[i];
+    tok[i] = m.token;
+    dptr[i] = m.dense;
+  }
+  for (int t = 0; t < T; ++t) {
+    uint32_t run = 0;
+    for (int i = 0; i < M; ++i) {
+      const Msg& m = h->fifo[i];
+      moff[(size_t)t * (M + 1) + i] = run;
+      run += (uint32_t)m.n[t];
+      iptr[(size_t)t * M + i] = m.ids[t];
+      rptr[(size_t)t * M + i] = m.rows[t];
+    }
+    moff[(size_t)t * (M + 1) + M] = run;
+  }
+  for (int t = 0; t <= T; ++t) nb[t] = nbase[t];
+  GBA_CUDA(h, cudaMemcpyAsync(h->d_meta, hp, h->meta_bytes, cudaMemcpyHostToDevice, h->stream));
+  cudaEventRecord(h->meta_ev[slot], h->stream);
+
+  StepArgs a{};
+  a.k = h->k;
+  a.M = M;
+  a.T = T;
+  a.N = N;
+  a.iota = h->st.iota;
+  a.row_staleness = h->st.row_staleness;
+  a.sparse_den = h->st.sparse_denominator;
+  a.tokens = (const int64_t*)(h->d_meta + o_tok);
+  a.dense_ptr = (const float* const*)(h->d_meta + o_dense);
+  a.msg_off = (const uint32_t*)(h->d_meta + o_off);
+  a.ids_ptr = (const int64_t* const*)(h->d_meta + o_ids);
+  a.rows_ptr = (const float* const*)(h->d_meta + o_rows);
+  a.nbase = (const int64_t*)(h->d_meta + o_nbase);
+  a.tinfo = h->d_tinfo;
+
+  // ---- K1: message weights (Eq. (1)); clears the per-step scratch
+  {
+    Timed tm(h, GBA_K_WEIGHTS, h->stream);
+    launch_weights(a, h->sc, h->d_stats, MAX_PASSES * 256, h->stream);
+  }
+  // ---- K5 on the side stream, concurrently with the sparse chain
+  if (h->D > 0) {
+    const double p1 = h->dbpow1 * (double)h->dense_opt.beta1;
+    const double p2 = h->dbpow2 * (double)h->dense_opt.beta2;
+    DenseArgs da{h->dw, h->ds0, h->ds1, h->D, M, make_opt_step(h->dense_opt, p1, p2)};
+    cudaEventRecord(h->ev_fork, h->stream);
+    cudaStreamWaitEvent(h->side, h->ev_fork, 0);
+    {
+      Timed tm(h, GBA_K_DENSE, h->side);
+      launch_dense(a, da, h->sc, h->sink, h->wait_ns, h->num_sms, h->side);
+    }
+    cudaEventRecord(h->ev_join, h->side);
+    h->dbpow1 = p1;
+    h->dbpow2 = p2;
+  }
+  // ---- K2 sort, K3+K4 segment-sum and row update
+  int final_buf = 0;
+  if (N > 0) {
+    {
+      Timed tm(h, GBA_K_SORT_HIST, h->stream);
+      int grid = (int)std::min<int64_t>((N + 255) / 256, (int64_t)h->num_sms * 8);
+      launch_sort_histogram(a, h->passes, h->sc, h->sink, std::max(grid, 1), h->stream);
+    }
+    const uint32_t* kin = nullptr;
+    const uint32_t* vin = nullptr;
+    for (int p = 0; p < h->passes; ++p) {
+      const int ob = p & 1;
+      if (++h->epoch == 0u) h->epoch = 1u;
+      Timed tm(h, GBA_K_SORT_PASS, h->stream);
+      launch_onesweep(a, p == 0, p, kin, vin, h->d_keys[ob], h->d_vals[ob], h->sc, h->d_status,
+                      h->epoch, h->sink, h->wait_ns, h->stream);
+      kin = h->d_keys[ob];
+      vin = h->d_vals[ob];
+      final_buf = ob;
+    }
+    for (int t = 0; t < T; ++t) {
+      const int64_t Nt = nbase[t + 1] - nbase[t];
+      if (Nt == 0) continue;
+      TableState& ts = h->tables[t];
+      const double p1 = ts.bpow1 * (double)ts.desc.opt.beta1;
+      const double p2 = ts.bpow2 * (double)ts.desc.opt.beta2;
+      SegTable tb{};
+      tb.w = ts.w;
+      tb.s0 = ts.s0;
+      tb.s1 = ts.s1;
+      tb.ver = ts.ver;
+      tb.d = ts.desc.dim;
+      tb.t = t;
+      tb.key_base = ts.key_base;
+      tb.rows = ts.desc.rows;
+      tb.pos_begin = nbase[t];
+      tb.pos_end = nbase[t + 1];
+      tb.opt = make_opt_step(ts.desc.opt, p1, p2);
+      const int64_t target = (int64_t)h->num_sms * 32;
+      int64_t range = (Nt + target - 1) / target;
+      range = std::max<int64_t>(64, (range + 63) / 64 * 64);
+      const int64_t n_warps = (Nt + range - 1) / range;
+      uint32_t* dc = h->debug ? h->d_dbg_count : nullptr;
+      uint32_t* dk = h->debug ? h->d_dbg_kept : nullptr;
+      {
+        Timed tm(h, GBA_K_SEGSUM, h->stream);
+        launch_segsum(a, tb, h->d_keys[final_buf], h->d_vals[final_buf], range, n_warps, h->rec,
+                      h->d_stats, dc, dk, h->sink, h->num_sms, h->stream);
+      }
+      {
+        Timed tm(h, GBA_K_FIXUP, h->stream);
+        launch_fixup(a, tb, n_warps, h->rec, h->d_stats, dc, dk, h->sink, h->stream);
+      }
+    }
+  }
+  // Adam step counts advance every global step, whether or not a row moved.
+  for (auto& ts : h->tables) {
+    ts.bpow1 *= (double)ts.desc.opt.beta1;
+    ts.bpow2 *= (double)ts.desc.opt.beta2;
+  }
+  if (h->D > 0) cudaStreamWaitEvent(h->stream, h->ev_join, 0);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    h->failed = true;
+    h->fail_code = cuda_fail(h, e, "kernel launch");
+    return h->fail_code;
+  }
+
+  // ---- pop the applied messages
+  for (int i = 0; i < M; ++i) {
+    Msg& m = h->fifo.front();
+    if (m.copied) {
+      for (int t = 0; t < T; ++t)
+        if (m.n[t] > 0) h->tables[t].arena.release_through(m.arena_v[t] + m.n[t]);
+      if (h->D > 0) {
+        h->slot_head = (h->slot_head + 1) % h->max_buf;
+        h->slot_count--;
+      }
+    }
+    h->fifo.pop_front();
+  }
+  h->k += 1;
+  h->have_last = true;
+  h->last_N = N;
+  h->last_buf = final_buf;
+  h->last_M = M;
+  return 1;
+}
+
+int64_t gba_pull_version(gba_handle* h) { return h ? h->k : -1; }
+
+gba_status gba_sync(gba_handle* h) {
+  if (!h) return GBA_E_ARG;
+  if (h->failed) return h->fail_code == GBA_OK ? GBA_E_STATE : h->fail_code;
+  cudaSetDevice(h->device);
+  return poll_device_error(h, true);
+}
+
+gba_status gba_get_table(gba_handle* h, int32_t t, float** w, float** slot0, float** slot1,
+                         int32_t** ver) {
+  if (!h || t < 0 || t >= h->T) return GBA_E_ARG;
+  const TableState& ts = h->tables[t];
+  if (w) *w = ts.w;
+  if (slot0) *slot0 = ts.s0;
+  if (slot1) *slot1 = ts.s1;
+  if (ver) *ver = ts.ver;
+  return GBA_OK;
+}
+
+gba_status gba_get_dense(gba_handle* h, float** w, float** slot0, float** slot1) {
+  if (!h) return GBA_E_ARG;
+  if (w) *w = h->dw;
+  if (slot0) *slot0 = h->ds0;
+  if (slot1) *slot1 = h->ds1;
+  return GBA_OK;
+}
+
+gba_status gba_stats(gba_handle* h, gba_stats_t* out) {
+  if (!h || !out) return GBA_E_ARG;
+  cudaSetDevice(h->device);
+  cudaStreamSynchronize(h->side);
+  DevStats s{};
+  GBA_CUDA(h, cudaMemcpyAsync(&s, h->d_stats, sizeof s, cudaMemcpyDeviceToHost, h->stream));
+  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  out->steps = (int64_t)s.steps;
+  out->msgs_kept = (int64_t)s.msgs_kept;
+  out->msgs_dropped = (int64_t)s.msgs_dropped;
+  out->dense_stale_sum = (int64_t)s.dense_stale_sum;
+  out->dense_stale_max = (int64_t)s.dense_stale_max;
+  out->pairs = (int64_t)s.pairs;
+  out->pairs_dropped = (int64_t)s.pairs_dropped;
+  out->row_stale_sum = (int64_t)s.row_stale_sum;
+  out->row_stale_max = (int64_t)s.row_stale_max;
+  out->occurrences = (int64_t)s.occurrences;
+  out->rows_touched = (int64_t)s.rows_touched;
+  out->rows_applied = (int64_t)s.rows_applied;
+  out->occurrences_kept = (int64_t)s.occ_kept;
+  return GBA_OK;
+}
+
+const char* gba_last_error(gba_handle* h) { return h ? h->last_error.c_str() : ""; }
+
+void gba_destroy(gba_handle* h) {
+  if (!h) return;
+  free_all(h);
+  delete h;
+}
+
+gba_status gba_set_timing(gba_handle* h, int32_t on) {
+  if (!h) return GBA_E_ARG;
+  cudaStreamSynchronize(h->side);
+  cudaStreamSynchronize(h->stream);
+  collect_timing(h);
+  h->times = gba_kernel_times_t{};
+  h->timing = on != 0;
+  return GBA_OK;
+}
+
+gba_status gba_kernel_times(gba_handle* h, gba_kernel_times_t* out) {
+  if (!h || !out) return GBA_E_ARG;
+  cudaSetDevice(h->device);
+  cudaStreamSynchronize(h->side);
+  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  collect_timing(h);
+  *out = h->times;
+  return GBA_OK;
+}
+
+gba_status gba_set_debug(gba_handle* h, int32_t on) {
+  if (!h) return GBA_E_ARG;
+  h->debug = on != 0;
+  return GBA_OK;
+}
+
+gba_status gba_debug_segments(gba_handle* h, int64_t cap, int32_t* table, int64_t* row,
+                              int64_t* count, int64_t* kept, int64_t* n_unique) {
+  if (!h || !n_unique) return GBA_E_ARG;
+  if (!h->have_last || !h->debug || !h->d_dbg_count)
+    return set_err(h, GBA_E_STATE, "no debug record of a step (enable debug before the step)");
+  cudaSetDevice(h->device);
+  cudaStreamSynchronize(h->side);
+  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  const int64_t N = h->last_N;
+  std::vector<uint32_t> keys(N), cnt(N), kp(N);
+  if (N > 0) {
+    GBA_CUDA(h, cudaMemcpy(keys.data(), h->d_keys[h->last_buf], N * 4, cudaMemcpyDeviceToHost));
+    GBA_CUDA(h, cudaMemcpy(cnt.data(), h->d_dbg_count, N * 4, cudaMemcpyDeviceToHost));
+    GBA_CUDA(h, cudaMemcpy(kp.data(), h->d_dbg_kept, N * 4, cudaMemcpyDeviceToHost));
+  }
+  int64_t u = 0;
+  for (int64_t i = 0; i < N; ++i) {
+    if (i > 0 && keys[i] == keys[i - 1]) continue;
+    if (u < cap) {
+      int t = 0;
+      while (t + 1 < h->T && keys[i] >= h->tables[t + 1].key_base) ++t;
+      if (table) table[u] = t;
+      if (row) row[u] = (int64_t)(keys[i] - h->tables[t].key_base);
+      if (count) count[u] = cnt[i];
+      if (kept) kept[u] = kp[i];
+    }
+    ++u;
+  }
+  *n_unique = u;
+  return u > cap ? set_err(h, GBA_E_ARG, "capacity too small") : GBA_OK;
+}
+
+gba_status gba_debug_sorted(gba_handle* h, int64_t cap, uint32_t* keys, uint32_t* occ,
+                            int64_t* n) {
+  if (!h || !n) return GBA_E_ARG;
+  if (!h->have_last) return set_err(h, GBA_E_STATE, "no step applied yet");
+  cudaSetDevice(h->device);
+  cudaStreamSynchronize(h->side);
+  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  *n = h->last_N;
+  if (h->last_N > cap) return set_err(h, GBA_E_ARG, "capacity too small");
+  if (h->last_N > 0) {
+    if (keys)
+      GBA_CUDA(h, cudaMemcpy(keys, h->d_keys[h->last_buf], h->last_N * 4, cudaMemcpyDeviceToHost));
+    if (occ)
+      GBA_CUDA(h, cudaMemcpy(occ, h->d_vals[h->last_buf], h->last_N * 4, cudaMemcpyDeviceToHost));
+  }
+  return GBA_OK;
+}
+
+gba_status gba_debug_keep(gba_handle* h, int32_t cap, int32_t* keep, int32_t* M) {
+  if (!h || !M) return GBA_E_ARG;
+  if (!h->have_last) return set_err(h, GBA_E_STATE, "no step applied yet");
+  cudaSetDevice(h->device);
+  cudaStreamSynchronize(h->side);
+  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  *M = h->last_M;
+  if (h->last_M > cap) return set_err(h, GBA_E_ARG, "capacity too small");
+  if (keep && h->last_M > 0)
+    GBA_CUDA(h, cudaMemcpy(keep, h->sc.keep, h->last_M * 4, cudaMemcpyDeviceToHost));
+  return GBA_OK;
+}
+
+gba_status gba_debug_set_wait_limit(gba_handle* h, int64_t ns) {
+  if (!h || ns < 0) return GBA_E_ARG;
+  h->wait_ns = ns;
+  return GBA_OK;
+}
+
+gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream) {
+  if (limit_ns < 0 || limit_ns > 10000000000ll) return GBA_E_ARG;
+  uint32_t* d = nullptr;
+  if (cudaMalloc(&d, 2 * sizeof(uint32_t)) != cudaSuccess) return GBA_E_OOM;
+  uint32_t result = 0;
+  const int rc = launch_wait_selftest(limit_ns, (cudaStream_t)cuda_stream, d, &result);
+  cudaFree(d);
+  if (rc != 0) return GBA_E_CUDA;
+  return result ? GBA_E_DEVICE_TIMEOUT : GBA_OK;
+}
+
+const char* gba_version_string(void) { return "libgba 0.1 (sm_103a)"; }
+
+}  // extern "C"

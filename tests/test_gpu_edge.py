@@ -1,0 +1,315 @@
+"""Edge cases of the CUDA path against the CPU oracle, and its error handling
+(needs a GPU).  No case here faults or hangs the device: bad ids are caught by
+the kernels' own range checks, waits are bounded."""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2205_11048_gb300 import binding as B
+from paper_2205_11048_gb300 import workload as W
+from tests import _harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+
+
+def msg(token, ids_per_table, dims, D, B_=1, scale=0.01, gen=None, dtype_ids=torch.int64):
+    gen = gen or torch.Generator(device="cuda").manual_seed(token * 7 + len(ids_per_table))
+    ids = [torch.as_tensor(i, dtype=dtype_ids, device="cuda") for i in ids_per_table]
+    rows = [torch.randn(i.numel(), d, generator=gen, device="cuda") * scale
+            for i, d in zip(ids, dims)]
+    dense = torch.randn(D, generator=gen, device="cuda") * scale
+    return dict(token=token, local_batch=B_, ids=ids, rows=rows, dense=dense)
+
+
+def cfg_of(tables, D, G, dense_kind=W.ADAM, iota=1):
+    """tables: list of (rows, dim, id_mode, opt kind)."""
+    tcs = tuple(W.TableCfg(r, d, 1, 0, 1.1, mode, W.OptCfg(kind, 0.01 if kind == 0 else 0.001))
+                for (r, d, mode, kind) in tables)
+    return W.WorkloadCfg("edge", M=G, B=1, tables=tcs, D=D,
+                         dense_opt=W.OptCfg(dense_kind, 0.01 if dense_kind == 0 else 0.001),
+                         stale=W.StaleCfg("fresh"), iota=iota, seed=3)
+
+
+def run_custom(cfg, steps, rule=None, max_buf=64, max_ids=None, by_ref=False, tol=H.TOL_ONE_STEP):
+    """steps: list of lists of message dicts; every step must trigger exactly once."""
+    tables = [(tb.rows, tb.dim, tb.id_mode, max_ids or 4096, H.opt_desc(tb.opt))
+              for tb in cfg.tables]
+    rule = rule or dict(iota=cfg.iota)
+    g = B.GBA(tables, cfg.D, H.opt_desc(cfg.dense_opt), cfg.G, max_buf, seed=cfg.seed, **rule)
+    g.set_debug(True)
+    orc = H.make_oracle(cfg, rule=rule)
+    stats = {}
+    for batch in steps:
+        for m in batch:
+            (g.push_ref if by_ref else g.push)(m["token"], m["ids"], m["rows"], m["dense"],
+                                               m["local_batch"])
+            orc.push(H.to_oracle(m))
+        a, b = g.try_apply(), orc.try_apply()
+        assert a == b == 1
+        H.accumulate_stats(stats, orc.last_stats, orc)
+        if cfg.tables:
+            H.compare_segments(g, orc, True)
+        H.compare_state(g, orc, tol)
+    g.sync()
+    H.compare_stats(g, stats)
+    return g, orc
+
+
+def test_hand_example_matches_golden_exactly():
+    """The hand-worked golden example, through the CUDA path: exact values."""
+    from tests import _pins
+    gj = _pins.load_golden()["adagrad"]
+    F = _pins.F
+    lr, acc0 = F(gj["table"]["lr"]), F(gj["table"]["init_acc"])
+    tables = [(4, 2, 0, 8, B.opt_desc(0, lr, acc0))]
+    g = B.GBA(tables, 2, B.opt_desc(0, lr, acc0), 2, 8, iota=gj["iota"], seed=12345)
+    w0 = g.table(0)[0].cpu().numpy().astype(np.float64)
+    dw0 = g.dense()[0].cpu().numpy().astype(np.float64)
+    for step in gj["steps"]:
+        for m in step["messages"]:
+            ids = torch.tensor(m["ids"], dtype=torch.int64, device="cuda")
+            rows = torch.tensor(m["rows"], dtype=torch.float32, device="cuda")
+            g.push(m["token"], [ids], [rows], torch.tensor(m["dense"], dtype=torch.float32,
+                                                           device="cuda"), m["B"])
+        assert g.try_apply() == 1
+        e = step["expect"]
+        assert g.keep().tolist() == e["keep"]
+        w, s0, _, ver = g.table(0)
+        for r in range(4):
+            assert (w[r].cpu().numpy().astype(np.float64) - w0[r]).tolist() == \
+                [F(v) for v in e["dw"][str(r)]]
+            assert s0[r].cpu().numpy().astype(np.float64).tolist() == \
+                [F(v) for v in e["acc"][str(r)]]
+        assert ver.cpu().tolist() == e["ver"]
+        dw, ds0, _ = g.dense()
+        assert (dw.cpu().numpy().astype(np.float64) - dw0).tolist() == \
+            [F(v) for v in e["dense_dw"]]
+        assert ds0.cpu().numpy().astype(np.float64).tolist() == [F(v) for v in e["dense_acc"]]
+    g.close()
+
+
+@pytest.mark.parametrize("dim", [1, 3, 4, 8, 19, 24, 64, 128, 200, 256])
+@pytest.mark.parametrize("kind", [0, 1])
+def test_row_widths_and_optimizers(dim, kind):
+    rng = np.random.default_rng(dim * 10 + kind)
+    cfg = cfg_of([(997, dim, 0, kind)], D=33, G=3, iota=1)
+    steps = []
+    for k in range(3):
+        batch = []
+        for m in range(3):
+            n = int(rng.integers(0, 300))
+            ids = rng.zipf(1.3, n) % 997
+            tok = max(0, k - int(rng.integers(0, 3)))
+            batch.append(msg(tok, [ids], [dim], 33))
+        steps.append(batch)
+    run_custom(cfg, steps)
+
+
+def test_empty_messages_and_empty_steps():
+    cfg = cfg_of([(50, 4, 0, 0), (30, 8, 0, 1)], D=5, G=3)
+    steps = [
+        [msg(0, [[], []], [4, 8], 5), msg(0, [[1, 2], []], [4, 8], 5), msg(0, [[], [7]], [4, 8], 5)],
+        [msg(1, [[], []], [4, 8], 5)] * 3,            # no ids at all in the step
+        [msg(2, [[3] * 500, []], [4, 8], 5), msg(2, [[], []], [4, 8], 5),
+         msg(2, [[3], [29]], [4, 8], 5)],
+    ]
+    run_custom(cfg, steps)
+
+
+def test_everything_dropped():
+    """All messages beyond iota: dense still steps (Adam moments move), no row moves."""
+    cfg = cfg_of([(40, 4, 0, 1)], D=9, G=2, iota=0)
+    steps = [[msg(0, [[1, 2]], [4], 9), msg(0, [[2, 3]], [4], 9)],
+             [msg(1, [[5]], [4], 9), msg(1, [[6]], [4], 9)],
+             [msg(0, [[1, 7]], [4], 9), msg(0, [[2]], [4], 9)]]   # staleness 2 > 0
+    g, orc = run_custom(cfg, steps)
+    assert orc.last_keep.tolist() == [0, 0]
+
+
+def test_single_message_steps_and_token_ahead():
+    cfg = cfg_of([(20, 4, 0, 0)], D=4, G=1, iota=0)
+    steps = [[msg(0, [[1]], [4], 4)], [msg(5, [[1, 1, 2]], [4], 4)], [msg(2, [[2]], [4], 4)]]
+    run_custom(cfg, steps)
+
+
+@pytest.mark.parametrize("rule", [dict(iota=1, row_staleness=1),
+                                  dict(iota=1, sparse_denominator=1),
+                                  dict(iota=1, sparse_denominator=2),
+                                  dict(iota=O.INT32_MAX)])
+def test_rule_options(rule):
+    rng = np.random.default_rng(4)
+    cfg = cfg_of([(300, 8, 0, 0)], D=17, G=4)
+    steps = []
+    for k in range(5):
+        steps.append([msg(max(0, k - int(rng.integers(0, 4))), [rng.integers(0, 300, 50)], [8], 17)
+                      for _ in range(4)])
+    run_custom(cfg, steps, rule=rule)
+
+
+def test_modulo_negative_ids():
+    rng = np.random.default_rng(8)
+    cfg = cfg_of([(1009, 16, 1, 0)], D=8, G=2)
+    steps = [[msg(0, [rng.integers(-2**62, 2**62, 400)], [16], 8) for _ in range(2)]
+             for _ in range(2)]
+    run_custom(cfg, steps)
+
+
+def test_varying_local_batches_overshoot():
+    """Apply when the buffered local batches reach G; the shortest prefix is popped."""
+    cfg = cfg_of([(64, 4, 0, 0)], D=4, G=10)
+    a = [msg(0, [[1]], [4], 4, B_=3), msg(0, [[2]], [4], 4, B_=3), msg(0, [[1]], [4], 4, B_=5)]
+    tables = [(64, 4, 0, 16, B.opt_desc())]
+    g = B.GBA(tables, 4, B.opt_desc(1, 0.001), 10, 8, iota=1, seed=3)
+    orc = H.make_oracle(cfg)
+    for m in a[:2]:
+        g.push(m["token"], m["ids"], m["rows"], m["dense"], m["local_batch"])
+        orc.push(H.to_oracle(m))
+    assert g.try_apply() == 0 and orc.try_apply() == 0
+    extra = msg(0, [[9]], [4], 4, B_=7)
+    for m in (a[2], extra):
+        g.push(m["token"], m["ids"], m["rows"], m["dense"], m["local_batch"])
+        orc.push(H.to_oracle(m))
+    assert g.try_apply() == 1 and orc.try_apply() == 1
+    H.compare_state(g, orc, H.TOL_ONE_STEP)
+    assert g.try_apply() == 0 and orc.try_apply() == 0   # 7 < 10 buffered
+    g.close()
+
+
+def test_hot_row_spanning_many_warps():
+    """One row with 200K occurrences in a step: partial sums cross many warp
+    ranges and are stitched by the fixup kernel in order."""
+    gen = torch.Generator(device="cuda").manual_seed(1)
+    cfg = cfg_of([(5000, 16, 0, 1)], D=4, G=4, iota=2)
+    steps = []
+    for k in range(2):
+        batch = []
+        for m in range(4):
+            hot = torch.full((50_000,), 17, dtype=torch.int64, device="cuda")
+            cold = torch.randint(0, 5000, (3000,), generator=gen, device="cuda")
+            ids = torch.cat([hot[:25_000], cold, hot[25_000:]])
+            batch.append(msg(max(0, k - m % 3), [ids.cpu().numpy()], [16], 4))
+        steps.append(batch)
+    run_custom(cfg, steps, max_ids=60_000)
+
+
+def test_dense_only_and_tables_only():
+    cfg = cfg_of([], D=1031, G=2)
+    run_custom(cfg, [[msg(0, [], [], 1031), msg(0, [], [], 1031)]] * 2)
+    cfg = cfg_of([(100, 4, 0, 0)], D=0, G=2)
+    run_custom(cfg, [[msg(0, [[1, 2]], [4], 0), msg(0, [[2]], [4], 0)]] * 2)
+
+
+@pytest.mark.parametrize("D", [1, 2, 3, 4, 5, 1023, 1024, 1025, 4097, 100_003])
+def test_dense_sizes(D):
+    cfg = cfg_of([(10, 4, 0, 0)], D=D, G=3)
+    run_custom(cfg, [[msg(0, [[1]], [4], D), msg(0, [[]], [4], D), msg(0, [[2]], [4], D)],
+                     [msg(1, [[1]], [4], D), msg(0, [[3]], [4], D), msg(1, [[]], [4], D)]],
+               by_ref=True)
+
+
+def test_ragged_sort_sizes():
+    """Step sizes around the sort tile (4096) and the segment round (64)."""
+    rng = np.random.default_rng(2)
+    for n in (1, 63, 64, 65, 4095, 4096, 4097, 12289):
+        cfg = cfg_of([(70_000, 8, 0, 0)], D=4, G=1)
+        run_custom(cfg, [[msg(0, [rng.integers(0, 70_000, n)], [8], 4)]], max_ids=n)
+
+
+# ---------------------------------------------------------------------------
+# errors
+
+def test_id_out_of_range_fails_the_step_without_touching_state():
+    tables = [(10, 4, 0, 8, B.opt_desc())]
+    g = B.GBA(tables, 4, B.opt_desc(), 1, 4, seed=1)
+    w_before = _raw_table_w(g, 0)
+    d_before = _raw_dense(g)
+    m = msg(0, [[3, 10]], [4], 4)   # id 10 is outside [0, 10)
+    g.push(m["token"], m["ids"], m["rows"], m["dense"], 1)
+    rc = g.L.gba_try_apply(g.h)
+    if rc == 1:
+        rc = g.L.gba_sync(g.h)
+    assert rc == B.GBA_E_ID_RANGE
+    assert g.L.gba_try_apply(g.h) == B.GBA_E_STATE
+    torch.cuda.synchronize()
+    assert torch.equal(_raw_table_w(g, 0), w_before)
+    assert torch.equal(_raw_dense(g), d_before)
+    g.close()
+
+
+def _raw_table_w(g, t):
+    w, s0, s1, v = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p()
+    g.L.gba_get_table(g.h, t, ctypes.byref(w), ctypes.byref(s0), ctypes.byref(s1),
+                      ctypes.byref(v))
+    torch.cuda.synchronize()
+    n = g.rows[t] * g.dims[t]
+    return B._copy_device(w.value, n, torch.float32)
+
+
+def _raw_dense(g):
+    w, s0, s1 = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_void_p()
+    g.L.gba_get_dense(g.h, ctypes.byref(w), ctypes.byref(s0), ctypes.byref(s1))
+    torch.cuda.synchronize()
+    return B._copy_device(w.value, g.D, torch.float32)
+
+
+def test_push_validation_and_full_buffer():
+    tables = [(10, 4, 0, 3, B.opt_desc())]
+    g = B.GBA(tables, 4, B.opt_desc(), 100, 2, seed=1)
+    m = msg(0, [[1, 2]], [4], 4)
+    L, h = g.L, g.h
+    good = [B.gba_sparse_grad(m["ids"][0].data_ptr(), 2, m["rows"][0].data_ptr())]
+    too_many = [B.gba_sparse_grad(m["ids"][0].data_ptr(), 4, m["rows"][0].data_ptr())]
+    assert B.gba_push(h, -1, good, m["dense"].data_ptr(), 1) == B.GBA_E_ARG
+    assert B.gba_push(h, 0, good, m["dense"].data_ptr(), 0) == B.GBA_E_ARG
+    assert B.gba_push(h, 0, too_many, m["dense"].data_ptr(), 1) == B.GBA_E_ARG
+    assert B.gba_push(h, 0, good, None, 1) == B.GBA_E_ARG
+    assert B.gba_push_ref(h, 0, good, m["dense"].data_ptr() + 4, 1) == B.GBA_E_ARG  # misaligned
+    assert B.gba_push(h, 0, good, m["dense"].data_ptr(), 1) == B.GBA_OK
+    assert B.gba_push(h, 0, good, m["dense"].data_ptr(), 1) == B.GBA_OK
+    assert B.gba_push(h, 0, good, m["dense"].data_ptr(), 1) == B.GBA_E_FULL
+    assert L.gba_try_apply(h) == 0
+    g.close()
+
+
+def test_bounded_wait_gives_up():
+    """A device wait on a flag nothing sets returns GBA_E_DEVICE_TIMEOUT and
+    the context stays usable."""
+    L = B.load()
+    assert L.gba_selftest_wait_timeout(2_000_000, None) == B.GBA_E_DEVICE_TIMEOUT
+    x = torch.ones(4, device="cuda")
+    assert float((x * 2).sum()) == 8.0
+
+
+def test_tiny_wait_limit_in_sort_is_reported_or_harmless():
+    """With a zero wait limit the onesweep look-back gives up whenever a
+    predecessor tile is not ready yet; the step then fails with
+    GBA_E_DEVICE_TIMEOUT (or succeeds if no tile had to wait).  No dense
+    parameters here, so only the sort's waits are exercised."""
+    rng = np.random.default_rng(0)
+    cfg = cfg_of([(200_000, 8, 0, 0)], D=0, G=1)
+    tables = [(200_000, 8, 0, 300_000, B.opt_desc())]
+    g = B.GBA(tables, 0, None, 1, 4, seed=1)
+    g.set_wait_limit(0)
+    m = msg(0, [rng.integers(0, 200_000, 300_000)], [8], 0)
+    g.push(m["token"], m["ids"], m["rows"], m["dense"], 1)
+    rc = g.L.gba_try_apply(g.h)
+    if rc == 1:
+        rc = g.L.gba_sync(g.h)
+    assert rc in (B.GBA_OK, B.GBA_E_DEVICE_TIMEOUT)
+    g.close()
+    # the device is still usable: a fresh handle runs a step
+    g2 = B.GBA(tables, 0, None, 1, 4, seed=1)
+    g2.push(m["token"], m["ids"], m["rows"], m["dense"], 1)
+    assert g2.try_apply() == 1
+    g2.sync()
+    g2.close()

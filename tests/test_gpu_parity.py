@@ -1,0 +1,87 @@
+"""CUDA path against the CPU oracle on the same seeded inputs (needs a GPU).
+
+Integer outputs (unique rows, per-row message and kept counts, message
+weights, tags, counters) must match exactly; floats within 1e-5 after each
+apply step and 1e-4 after 100 steps, with the per-tensor relative metric
+max |a-b| / max(|b|, 1e-3 max|b|)."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2205_11048_gb300 import workload as W
+from tests import _harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5])
+def test_reduced_configs_few_steps(n):
+    cfg = W.reduced(n)
+    H.run_parity(cfg, steps=4, tol=H.TOL_ONE_STEP)
+
+
+@pytest.mark.parametrize("n", [2, 3, 5])
+def test_reduced_configs_by_reference(n):
+    cfg = W.reduced(n)
+    H.run_parity(cfg, steps=3, tol=H.TOL_ONE_STEP, by_ref=True)
+
+
+@pytest.mark.parametrize("n", [1, 2, 3, 4, 5])
+def test_hundred_steps(n):
+    cfg = W.reduced(n)
+    if n == 3:  # multi-hot: keep the oracle's run short, fewer ids per message
+        cfg = W.replace(cfg, B=6)
+    H.run_parity(cfg, steps=100, tol=H.TOL_MANY_STEPS, check_every=25, by_ref=True)
+
+
+def test_config1_full_twenty_steps():
+    cfg = W.config(1)
+    H.run_parity(cfg, steps=cfg.steps, tol=H.TOL_MANY_STEPS, check_every=5)
+
+
+@pytest.mark.parametrize("n", [3, 5])
+def test_sort_is_a_stable_sort(n):
+    """The sorted keys and payloads are exactly a stable sort of the step's
+    (global row, occurrence) pairs."""
+    cfg = W.reduced(n)
+    g = H.make_gpu(cfg)
+    msgs = W.generate_step(cfg, 0, "cuda")
+    for m in msgs:
+        H.push_gpu(g, m)
+    assert g.try_apply() == 1
+    keys, occ = g.sorted_keys()
+    base = 0
+    want = []
+    for t, tb in enumerate(cfg.tables):
+        for m in msgs:
+            want.append(H.rows_of(cfg, t, m["ids"][t].cpu().numpy()) + base)
+        base += tb.rows
+    want = np.concatenate(want).astype(np.uint32)
+    order = np.argsort(want, kind="stable")
+    assert np.array_equal(keys, want[order])
+    assert np.array_equal(occ, order.astype(np.uint32))
+    g.close()
+
+
+def test_bit_identical_run_to_run():
+    cfg = W.reduced(3)
+    outs = []
+    for _ in range(2):
+        g = H.make_gpu(cfg)
+        for k in range(2):
+            for m in W.generate_step(cfg, k, "cuda"):
+                H.push_gpu(g, m)
+            g.try_apply()
+        w, s0, _, ver = g.table(0)
+        dw, ds0, ds1 = g.dense()
+        outs.append((w.cpu(), s0.cpu(), ver.cpu(), dw.cpu(), ds1.cpu()))
+        g.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
