@@ -141,6 +141,21 @@ def measured_traffic(kernel, workload):
     return e.get("dram_bytes_per_launch")
 
 
+def max_over_ranks(x: float, pg, device="cpu") -> float:
+    """The largest value of x over all ranks (x itself without a process group)."""
+    if pg is None:
+        return float(x)
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(steps_per_rank: int, world: int, max_elapsed_ms: float) -> float:
+    """Whole-job steps/s: every rank's steps over the slowest rank's time."""
+    return steps_per_rank * world / (max_elapsed_ms / 1e3)
+
+
 def dist_setup():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -312,13 +327,9 @@ def run_gba(args):
     g.sync()
     st1 = g.stats()
     delta = {key: st1[key] - st0[key] for key in st1}
-    if pg:
-        t = torch.tensor([el_ms], device="cuda")
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        el_ms = float(t.item())
+    el_ms = max_over_ranks(el_ms, pg, "cuda")
     ms_per_step = el_ms / args.steps
-    total_steps = args.steps * ws
-    value = total_steps / (el_ms / 1e3)
+    value = job_throughput(args.steps, ws, el_ms)
     launches = sum(kt[n][0] for n in kt if n != "init")
 
     # roofline of the dominant kernel class

@@ -736,8 +736,11 @@ int32_t gba_try_apply(gba_handle* h) {
     Timed tm(h, GBA_K_WEIGHTS, h->stream);
     launch_weights(a, h->sc, h->d_stats, MAX_PASSES * 256, h->stream);
   }
-  // ---- K5 on the side stream, concurrently with the sparse chain
-  if (h->D > 0) {
+  // ---- K5 on the side stream, concurrently with the sort and segment-sum.
+  // It is forked after the histogram kernel has validated every id, so a step
+  // that fails its id check leaves the dense parameters untouched too.
+  auto launch_dense_side = [&]() {
+    if (h->D <= 0) return;
     const double p1 = h->dbpow1 * (double)h->dense_opt.beta1;
     const double p2 = h->dbpow2 * (double)h->dense_opt.beta2;
     DenseArgs da{h->dw, h->ds0, h->ds1, h->D, M, make_opt_step(h->dense_opt, p1, p2)};
@@ -750,7 +753,7 @@ int32_t gba_try_apply(gba_handle* h) {
     cudaEventRecord(h->ev_join, h->side);
     h->dbpow1 = p1;
     h->dbpow2 = p2;
-  }
+  };
   // ---- K2 sort, K3+K4 segment-sum and row update
   int final_buf = 0;
   if (N > 0) {
@@ -759,6 +762,7 @@ int32_t gba_try_apply(gba_handle* h) {
       int grid = (int)std::min<int64_t>((N + 255) / 256, (int64_t)h->num_sms * 8);
       launch_sort_histogram(a, h->passes, h->sc, h->sink, std::max(grid, 1), h->stream);
     }
+    launch_dense_side();
     const uint32_t* kin = nullptr;
     const uint32_t* vin = nullptr;
     for (int p = 0; p < h->passes; ++p) {
@@ -806,6 +810,7 @@ int32_t gba_try_apply(gba_handle* h) {
       }
     }
   }
+  if (N == 0) launch_dense_side();
   // Adam step counts advance every global step, whether or not a row moved.
   for (auto& ts : h->tables) {
     ts.bpow1 *= (double)ts.desc.opt.beta1;

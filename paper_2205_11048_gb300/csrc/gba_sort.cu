@@ -24,6 +24,7 @@ constexpr int SORT_WARPS = SORT_THREADS / 32;
 constexpr int SORT_ITEMS = 16;
 constexpr int SORT_TILE = SORT_THREADS * SORT_ITEMS;
 constexpr int MAX_PASSES = 4;
+constexpr int LB_WIN = 8;  // look-back window
 
 // Look-back status word: [63:32] epoch of the launch, [31:30] flag, [29:0] count.
 constexpr unsigned long long FLAG_AGG = 1ull << 30;
@@ -31,13 +32,13 @@ constexpr unsigned long long FLAG_INCL = 2ull << 30;
 constexpr unsigned long long FLAG_MASK = 3ull << 30;
 constexpr unsigned long long COUNT_MASK = (1ull << 30) - 1;
 
-__device__ __forceinline__ unsigned long long ld_acquire_u64(const unsigned long long* p) {
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
   unsigned long long v;
-  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
   return v;
 }
-__device__ __forceinline__ void st_release_u64(unsigned long long* p, unsigned long long v) {
-  asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+__device__ __forceinline__ void st_relaxed_u64(unsigned long long* p, unsigned long long v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 __device__ __forceinline__ uint32_t ld_volatile_u32(const uint32_t* p) {
   return *(const volatile uint32_t*)p;
@@ -239,29 +240,47 @@ __global__ void __launch_bounds__(SORT_THREADS)
   const uint32_t tile_count = run;
   unsigned long long* my = status + (size_t)tile * RADIX + d;
   const unsigned long long ep = (unsigned long long)epoch << 32;
-  st_release_u64(my, ep | (tile == 0 ? FLAG_INCL : FLAG_AGG) | tile_count);
+  st_relaxed_u64(my, ep | (tile == 0 ? FLAG_INCL : FLAG_AGG) | tile_count);
 
   const uint32_t g_excl = block_excl_scan_256(sc.hist[pass * RADIX + d], s_tmp);
   const uint32_t t_excl = block_excl_scan_256(tile_count, s_tmp);
   s_tile_excl[d] = t_excl;
 
+  // Decoupled look-back over a window of LB_WIN predecessors at a time: the
+  // window's status words are read with independent loads, then consumed from
+  // the nearest tile backwards until an inclusive prefix is found.  The words
+  // are self-contained (no other data is published with them), so relaxed
+  // loads and stores suffice.
   uint32_t prefix = 0;
   if (tile > 0) {
     int64_t j = (int64_t)tile - 1;
     const uint64_t t0 = globaltimer_ns();
-    while (j >= 0) {
-      const unsigned long long v = ld_acquire_u64(status + (size_t)j * RADIX + d);
-      if ((v & ~0xFFFFFFFFull) == ep && (v & FLAG_MASK) != 0ull) {
-        prefix += (uint32_t)(v & COUNT_MASK);
-        if (v & FLAG_INCL) break;
-        --j;
-      } else if ((ld_volatile_u32(err.dev) & ERR_TIMEOUT) ||
-                 (int64_t)(globaltimer_ns() - t0) > wait_ns) {
+    bool done = false;
+    while (!done) {
+      unsigned long long v[LB_WIN];
+#pragma unroll
+      for (int i = 0; i < LB_WIN; ++i)
+        v[i] = (j - i >= 0) ? ld_relaxed_u64(status + (size_t)(j - i) * RADIX + d) : 0ull;
+      int used = 0;
+#pragma unroll
+      for (int i = 0; i < LB_WIN; ++i) {
+        if (done || used != i || j - i < 0) continue;
+        const unsigned long long x = v[i];
+        if ((x & ~0xFFFFFFFFull) != ep || (x & FLAG_MASK) == 0ull) continue;  // not ready
+        prefix += (uint32_t)(x & COUNT_MASK);
+        used = i + 1;
+        if (x & FLAG_INCL) done = true;
+      }
+      if (done) break;
+      j -= used;
+      if (j < 0) break;  // cannot happen: tile 0 publishes an inclusive prefix
+      if (used == 0 && ((ld_volatile_u32(err.dev) & ERR_TIMEOUT) ||
+                        (int64_t)(globaltimer_ns() - t0) > wait_ns)) {
         raise_error(err, ERR_TIMEOUT);
         break;
       }
     }
-    st_release_u64(my, ep | FLAG_INCL | ((prefix + tile_count) & COUNT_MASK));
+    st_relaxed_u64(my, ep | FLAG_INCL | ((prefix + tile_count) & COUNT_MASK));
   }
   s_out_base[d] = g_excl + prefix;
   __syncthreads();
