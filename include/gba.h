@@ -241,6 +241,39 @@ gba_status gba_debug_set_wait_limit(gba_handle* h, int64_t ns);
  */
 gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream);
 
+/*
+ * gba_sort_ids_static - sort one batch of ids by row without allocating.
+ *
+ * The paper has no counterpart to this entry point; it exists for callers that
+ * cannot allocate device memory when they need the sort, for example code that
+ * is being captured into a CUDA graph (an allocation is not a stream operation)
+ * or a runtime whose device memory is entirely reserved up front.  It runs the
+ * same histogram and onesweep radix-sort kernels as gba_try_apply, but takes
+ * its scratch from one fixed device array of GBA_STATIC_SORT_BYTES bytes that
+ * the library reserves when it is loaded; every GPU that loads the library
+ * keeps that array until the process exits.  The call allocates nothing.
+ *
+ * ids        n device int64 ids; row = id (id_mode DIRECT, 0 <= id < rows) or
+ *            (uint64)id % rows (MODULO).
+ * n          0 .. GBA_STATIC_SORT_MAX_IDS; larger n returns GBA_E_ARG.
+ * rows       1 .. 2^32 - 2.
+ * rows_out   n device uint32: the rows of the ids in ascending order.
+ * order_out  n device uint32: order_out[i] is the input index of rows_out[i];
+ *            equal rows keep their input order (stable).
+ * cuda_stream  the stream to run on (NULL: the legacy default stream); the call
+ *            returns after the work has finished on it, with GBA_OK,
+ *            GBA_E_ID_RANGE (a DIRECT id outside [0, rows)), GBA_E_DEVICE_TIMEOUT
+ *            or GBA_E_CUDA.
+ * The first call on a device, with that device current, looks up the array's
+ * device address; make that first call before any stream capture.  All calls
+ * share the one array and it keeps the previous call's contents (counters are
+ * cleared at the start of each call); calls whose work overlaps on the GPU race.
+ */
+#define GBA_STATIC_SORT_MAX_IDS (1 << 20)
+#define GBA_STATIC_SORT_BYTES 8917104
+gba_status gba_sort_ids_static(const int64_t* ids, int64_t n, int64_t rows, int32_t id_mode,
+                               uint32_t* rows_out, uint32_t* order_out, void* cuda_stream);
+
 /* gba_version_string - library build identification. */
 const char* gba_version_string(void);
 

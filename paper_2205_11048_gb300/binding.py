@@ -104,6 +104,8 @@ _SIGNATURES = {
     "gba_debug_set_wait_limit": (ctypes.c_int, [_P, ctypes.c_int64]),
     "gba_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int64, _P]),
     "gba_version_string": (ctypes.c_char_p, []),
+    "gba_sort_ids_static": (ctypes.c_int, [_P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32,
+                                           _P, _P, _P]),
 }
 
 _lib = None
