@@ -1,0 +1,218 @@
+// Internal declarations shared by the translation units of libgba.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace gba {
+
+// ---- device error word bits -------------------------------------------------
+constexpr uint32_t ERR_ID_RANGE = 1u;
+constexpr uint32_t ERR_TIMEOUT = 2u;
+constexpr uint32_t ERR_INTERNAL = 4u;
+
+// Where kernels report a failure: an atomic word in device memory plus a flag
+// in mapped pinned host memory the host can poll without synchronising.
+struct ErrSink {
+  uint32_t* dev;
+  volatile uint32_t* host;
+};
+
+__device__ __forceinline__ void raise_error(const ErrSink& e, uint32_t code) {
+  atomicOr(e.dev, code);
+  *e.host = 1u;
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ---- per-table static description (device copy) ----------------------------
+struct TableInfo {
+  int64_t V;
+  uint32_t key_base;  // first global key of the table
+  int32_t id_mode;    // 0 DIRECT, 1 MODULO
+};
+
+// ---- optimizer parameters of one parameter group for one step ---------------
+struct OptStep {
+  int32_t kind;  // 0 Adagrad, 1 Adam
+  float lr, b1, b2, eps;
+  float c1, c2;    // 1 - b1, 1 - b2 (float arithmetic)
+  float bc1, bc2;  // Adam bias corrections of this step
+};
+
+// Adagrad and Adam, one IEEE float operation at a time in a fixed order.
+__device__ __forceinline__ void opt_update(const OptStep& o, float& w, float& s0, float& s1,
+                                           float g) {
+  if (o.kind == 0) {
+    float gg = __fmul_rn(g, g);
+    float an = __fadd_rn(s0, gg);
+    float step = __fmul_rn(o.lr, g);
+    float den = __fsqrt_rn(an);
+    s0 = an;
+    w = __fsub_rn(w, __fdiv_rn(step, den));
+  } else {
+    float mn = __fadd_rn(__fmul_rn(o.b1, s0), __fmul_rn(o.c1, g));
+    float gg = __fmul_rn(g, g);
+    float vn = __fadd_rn(__fmul_rn(o.b2, s1), __fmul_rn(o.c2, gg));
+    float mhat = __fdiv_rn(mn, o.bc1);
+    float vhat = __fdiv_rn(vn, o.bc2);
+    float num = __fmul_rn(o.lr, mhat);
+    float den = __fadd_rn(__fsqrt_rn(vhat), o.eps);
+    s0 = mn;
+    s1 = vn;
+    w = __fsub_rn(w, __fdiv_rn(num, den));
+  }
+}
+
+// Error-free transformation of a + b (Knuth's TwoSum): s + e == a + b exactly.
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = __fadd_rn(a, b);
+  float bp = __fsub_rn(s, a);
+  float ap = __fsub_rn(s, bp);
+  e = __fadd_rn(__fsub_rn(a, ap), __fsub_rn(b, bp));
+}
+
+// Compensated accumulator: value = hi + lo.
+struct CSum {
+  float hi, lo;
+};
+__device__ __forceinline__ void csum_add(CSum& c, float x) {
+  float s, e;
+  two_sum(c.hi, x, s, e);
+  c.hi = s;
+  c.lo = __fadd_rn(c.lo, e);
+}
+__device__ __forceinline__ void csum_merge(CSum& c, float hi, float lo) {
+  float s, e;
+  two_sum(c.hi, hi, s, e);
+  c.hi = s;
+  c.lo = __fadd_rn(__fadd_rn(c.lo, lo), e);
+}
+__device__ __forceinline__ float csum_value(const CSum& c) { return __fadd_rn(c.hi, c.lo); }
+
+// ---- one global step, as seen by the kernels ---------------------------------
+// Passed by value to every kernel of a step; the arrays live in a device
+// buffer the host fills before the step.
+struct StepArgs {
+  int64_t k;
+  int32_t M;           // messages popped
+  int32_t T;           // tables
+  int64_t N;           // id occurrences over all tables
+  int32_t iota;
+  int32_t row_staleness;
+  int32_t sparse_den;
+  int32_t pad0;
+  const int64_t* tokens;          // [M]
+  const float* const* dense_ptr;  // [M]
+  const uint32_t* msg_off;        // [T][M+1] occurrence offsets within the table
+  const int64_t* const* ids_ptr;  // [T][M]
+  const float* const* rows_ptr;   // [T][M]
+  const int64_t* nbase;           // [T+1] first global occurrence of each table
+  const TableInfo* tinfo;         // [T]
+};
+
+// Per-step device scratch that K1 clears at the start of a step.
+struct StepScratch {
+  uint32_t* hist;          // [4][256] digit histograms of the key passes
+  uint32_t* tile_counter;  // [4] onesweep tile tickets
+  int32_t* keep;           // [M] message weights f
+  int32_t* kept_list;      // [M] indices of kept messages, in pop order
+  int32_t* n_kept;         // [1]
+};
+
+// Accumulated statistics (device).
+struct DevStats {
+  unsigned long long steps, msgs_kept, msgs_dropped, dense_stale_sum, dense_stale_max, pairs,
+      pairs_dropped, row_stale_sum, row_stale_max, occurrences, rows_touched, rows_applied,
+      occ_kept;
+};
+
+// The message that holds table-local occurrence x: the largest m in [0, M)
+// with off[m] <= x, given off[0] = 0 <= x < off[M] (empty messages repeat an
+// offset and are skipped by taking the largest such m).
+__device__ __forceinline__ int message_of(const uint32_t* off, int M, uint32_t x) {
+  int lo = 0, hi = M;  // off[lo] <= x < off[hi]
+  while (hi - lo > 1) {
+    int mid = (lo + hi) >> 1;
+    if (__ldg(off + mid) <= x)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  return lo;
+}
+
+// ---- launch wrappers (defined in the kernel translation units) ---------------
+void launch_weights(const StepArgs& a, StepScratch sc, DevStats* stats, int n_hist_words,
+                    cudaStream_t s);
+
+void launch_sort_histogram(const StepArgs& a, int passes, StepScratch sc, ErrSink err, int grid,
+                           cudaStream_t s);
+
+void launch_onesweep(const StepArgs& a, bool first, int pass, const uint32_t* keys_in,
+                     const uint32_t* vals_in, uint32_t* keys_out, uint32_t* vals_out,
+                     StepScratch sc, unsigned long long* status, uint32_t epoch, ErrSink err,
+                     int64_t wait_ns, cudaStream_t s);
+
+int sort_tiles(int64_t N);
+
+struct SegTable {
+  float* w;
+  float* s0;
+  float* s1;
+  int32_t* ver;
+  int32_t d;
+  int32_t t;
+  uint32_t key_base;
+  int32_t pad;
+  int64_t rows;                // V of the table
+  int64_t pos_begin, pos_end;  // range of the sorted array holding this table's keys
+  OptStep opt;
+};
+
+// Partial sums of rows that cross warp ranges: per warp range, slot 0 is the
+// part of a row that began in an earlier range, slot 1 the part of a row that
+// begins in this range and continues into the next.
+struct SegRecords {
+  float* hi;       // [W][2][d_max] compensated partial sums
+  float* lo;       // [W][2][d_max]
+  uint32_t* meta;  // [W][2][6]  type, x, c_all, c_kept, k_occ, head_pos
+};
+
+void launch_segsum(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
+                   const uint32_t* vals, int64_t range, int64_t n_warps, SegRecords rec,
+                   DevStats* stats, uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err,
+                   int num_sms, cudaStream_t s);
+
+void launch_fixup(const StepArgs& a, const SegTable& tb, int64_t n_warps, SegRecords rec,
+                  DevStats* stats, uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err,
+                  cudaStream_t s);
+
+struct DenseArgs {
+  float* w;
+  float* s0;
+  float* s1;
+  int64_t D;
+  int32_t M;
+  OptStep opt;
+};
+
+size_t dense_smem_bytes();
+cudaError_t configure_dense();
+void launch_dense(const StepArgs& a, const DenseArgs& da, StepScratch sc, ErrSink err,
+                  int64_t wait_ns, int num_sms, cudaStream_t s);
+
+void launch_init_table(float* w, float* s0, float* s1, int32_t* ver, int64_t rows, int32_t d,
+                       int32_t kind, float init_acc, uint64_t seed, uint64_t tag,
+                       cudaStream_t s);
+
+void launch_init_dense(float* w, float* s0, float* s1, int64_t D, int32_t kind, float init_acc,
+                       uint64_t seed, uint64_t tag, cudaStream_t s);
+
+int launch_wait_selftest(int64_t limit_ns, cudaStream_t s, uint32_t* d_word, uint32_t* result);
+
+}  // namespace gba

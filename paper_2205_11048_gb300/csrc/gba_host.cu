@@ -592,7 +592,7 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
     h->sc.n_kept = (int32_t*)p;
   }
   {
-    h->rec_warps = (int64_t)h->num_sms * 32 + 64;
+    h->rec_warps = (int64_t)h->num_sms * 64 + 64;
     const size_t nf = (size_t)h->rec_warps * 2 * h->d_max;
     if (!dev_alloc((void**)&h->rec.hi, nf * 4) || !dev_alloc((void**)&h->rec.lo, nf * 4) ||
         !dev_alloc((void**)&h->rec.meta, (size_t)h->rec_warps * 2 * 6 * 4))
@@ -793,16 +793,13 @@ int32_t gba_try_apply(gba_handle* h) {
       tb.pos_begin = nbase[t];
       tb.pos_end = nbase[t + 1];
       tb.opt = make_opt_step(ts.desc.opt, p1, p2);
-      const int64_t target = (int64_t)h->num_sms * 32;
-      int64_t range = (Nt + target - 1) / target;
-      range = std::max<int64_t>(64, (range + 63) / 64 * 64);
-      const int64_t n_warps = (Nt + range - 1) / range;
       uint32_t* dc = h->debug ? h->d_dbg_count : nullptr;
       uint32_t* dk = h->debug ? h->d_dbg_kept : nullptr;
+      int64_t n_warps = 0;
       {
         Timed tm(h, GBA_K_SEGSUM, h->stream);
-        launch_segsum(a, tb, h->d_keys[final_buf], h->d_vals[final_buf], range, n_warps, h->rec,
-                      h->d_stats, dc, dk, h->sink, h->num_sms, h->stream);
+        n_warps = launch_segsum(a, tb, h->d_keys[final_buf], h->d_vals[final_buf], h->rec,
+                                h->rec_warps, h->d_stats, dc, dk, h->sink, h->num_sms, h->stream);
       }
       {
         Timed tm(h, GBA_K_FIXUP, h->stream);

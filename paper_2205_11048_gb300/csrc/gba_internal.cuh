@@ -183,10 +183,12 @@ struct SegRecords {
   uint32_t* meta;  // [W][2][6]  type, x, c_all, c_kept, k_occ, head_pos
 };
 
-void launch_segsum(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
-                   const uint32_t* vals, int64_t range, int64_t n_warps, SegRecords rec,
-                   DevStats* stats, uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err,
-                   int num_sms, cudaStream_t s);
+// Launches the segment-sum + row update over table tb's range of the sorted
+// array; returns the number of warp ranges (for the fixup launch).
+int64_t launch_segsum(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
+                      const uint32_t* vals, SegRecords rec, int64_t max_warps, DevStats* stats,
+                      uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
+                      cudaStream_t s);
 
 void launch_fixup(const StepArgs& a, const SegTable& tb, int64_t n_warps, SegRecords rec,
                   DevStats* stats, uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err,

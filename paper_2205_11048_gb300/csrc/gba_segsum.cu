@@ -6,13 +6,16 @@
 //
 // Work is split by occurrences, not by rows, so Zipf-hot rows cost no more per
 // occurrence than cold ones.  Each warp owns a contiguous range of the sorted
-// array and walks it in rounds of 64 positions; within a round each lane group
-// (L lanes, one row-slice of 16-byte vectors per lane) sums a contiguous slice
-// of positions sequentially with compensated (TwoSum) float accumulation.
-// Rows that start and end inside a slice are applied by their group at once;
-// rows crossing slices are stitched in slice order across the warp; rows
+// array.  Lane l holds elements [l*EPL, (l+1)*EPL) of the row being summed, so
+// the walk over the positions is warp-uniform: the per-position metadata
+// (row pointer, head / kept / new-message flags) is computed by all lanes in
+// parallel for a round of 64 positions, then the warp streams through the
+// round's gradient rows eight at a time (loads issued before they are summed),
+// accumulating with compensated (TwoSum) float arithmetic.  A finished row's
+// aggregated gradient goes to a small per-warp queue in shared memory; the
+// queue is applied eight rows at a time, all state loads issued first.  Rows
 // crossing warp ranges leave partial sums in a record that the fixup kernel
-// combines in range order.  All orders are fixed, so results are bit-identical
+// combines in range order.  Every order is fixed, so results are bit-identical
 // run to run.
 #include "gba_internal.cuh"
 
@@ -20,23 +23,32 @@ namespace gba {
 
 namespace {
 
-constexpr int SEG_THREADS = 256;
-constexpr int SEG_WARPS = SEG_THREADS / 32;
-constexpr int RS = 64;  // positions per round
+constexpr int SEG_WARPS = 4;
+constexpr int SEG_THREADS = SEG_WARPS * 32;
+constexpr int RS = 32;  // positions per round: one per lane
+// finished rows per update batch: 8 rows of up to 64 floats, fewer wider ones
+template <int EPL>
+__host__ __device__ constexpr int pb_rows() { return EPL <= 2 ? 8 : (EPL == 4 ? 4 : 2); }
+template <int EPL>
+__host__ __device__ constexpr int queue_rows() { return pb_rows<EPL>(); }
+// dynamic shared memory of one block: staged rows and the finished-row queue
+template <int EPL>
+__host__ __device__ constexpr size_t seg_dyn_smem() {
+  return (size_t)SEG_WARPS * (RS + queue_rows<EPL>()) * 32 * EPL * sizeof(float);
+}
 
-constexpr uint32_t F_HEAD = 1u, F_KEEP = 2u, F_NEWMSG = 4u;
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void stage_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+constexpr int MSG_CACHE = 256;  // messages whose lookups are cached in shared memory
 
 // record types
 constexpr uint32_t REC_NONE = 0u, REC_PASS = 1u, REC_CLOSED = 2u, REC_OWNER = 3u;
 constexpr int REC_META = 6;  // type, x, c_all, c_kept, k_occ, head_pos
 
-struct PosMeta {
-  const float* row;  // gradient row of the occurrence
-  uint32_t key;
-  uint32_t m;        // message index
-  uint32_t flags;
-  uint32_t pad;
-};
 
 __device__ __forceinline__ uint32_t ld_volatile_u32(const uint32_t* p) {
   return *(const volatile uint32_t*)p;
@@ -49,47 +61,39 @@ __device__ __forceinline__ float row_denominator(int mode, uint32_t c_all, uint3
   return (float)den;
 }
 
-template <int VEC>
-struct Vec;
-template <>
-struct Vec<4> {
-  static __device__ __forceinline__ void load(const float* p, float* v) {
-    const float4 q = *reinterpret_cast<const float4*>(p);
-    v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
-  }
-  static __device__ __forceinline__ void store(float* p, const float* v) {
-    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
-  }
-};
-template <>
-struct Vec<1> {
-  static __device__ __forceinline__ void load(const float* p, float* v) { v[0] = *p; }
-  static __device__ __forceinline__ void store(float* p, const float* v) { *p = v[0]; }
-};
-
-// Apply the optimizer to this lane's slice of row x: element (e*L + l)*VEC + v.
-template <int VEC, int L, int EPL>
-__device__ __forceinline__ void apply_slice(const SegTable& tb, uint32_t x, int l,
-                                            const CSum* s, float den) {
-  const int d = tb.d;
-  const size_t rb = (size_t)x * (size_t)d;
+// EPL consecutive floats at p (vector access when VECOK: p is EPL*4-aligned).
+template <int EPL, bool VECOK>
+__device__ __forceinline__ void load_lane(const float* p, int n_valid, float* v) {
+  if constexpr (VECOK && EPL == 1) {
+    v[0] = *p;
+  } else if constexpr (VECOK && EPL == 2) {
+    const float2 q = *reinterpret_cast<const float2*>(p);
+    v[0] = q.x; v[1] = q.y;
+  } else if constexpr (VECOK && EPL % 4 == 0) {
 #pragma unroll
-  for (int e = 0; e < EPL; ++e) {
-    const int idx = (e * L + l) * VEC;
-    if (idx < d) {
-      float w[VEC], s0[VEC], s1[VEC];
-      Vec<VEC>::load(tb.w + rb + idx, w);
-      Vec<VEC>::load(tb.s0 + rb + idx, s0);
-      if (tb.opt.kind == 1) Vec<VEC>::load(tb.s1 + rb + idx, s1);
-#pragma unroll
-      for (int v = 0; v < VEC; ++v) {
-        const float g = __fdiv_rn(csum_value(s[e * VEC + v]), den);
-        opt_update(tb.opt, w[v], s0[v], s1[v], g);
-      }
-      Vec<VEC>::store(tb.w + rb + idx, w);
-      Vec<VEC>::store(tb.s0 + rb + idx, s0);
-      if (tb.opt.kind == 1) Vec<VEC>::store(tb.s1 + rb + idx, s1);
+    for (int i = 0; i < EPL; i += 4) {
+      const float4 q = *reinterpret_cast<const float4*>(p + i);
+      v[i] = q.x; v[i + 1] = q.y; v[i + 2] = q.z; v[i + 3] = q.w;
     }
+  } else {
+#pragma unroll
+    for (int i = 0; i < EPL; ++i) v[i] = i < n_valid ? p[i] : 0.f;
+  }
+}
+template <int EPL, bool VECOK>
+__device__ __forceinline__ void store_lane(float* p, int n_valid, const float* v) {
+  if constexpr (VECOK && EPL == 1) {
+    *p = v[0];
+  } else if constexpr (VECOK && EPL == 2) {
+    *reinterpret_cast<float2*>(p) = make_float2(v[0], v[1]);
+  } else if constexpr (VECOK && EPL % 4 == 0) {
+#pragma unroll
+    for (int i = 0; i < EPL; i += 4)
+      *reinterpret_cast<float4*>(p + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+  } else {
+#pragma unroll
+    for (int i = 0; i < EPL; ++i)
+      if (i < n_valid) p[i] = v[i];
   }
 }
 
@@ -97,46 +101,58 @@ struct RunCounts {
   uint32_t c_all, c_kept, k_occ;
 };
 
-// Everything that happens when a row's run is complete.
-template <int VEC, int L, int EPL>
-__device__ __forceinline__ void finalize_row(const StepArgs& a, const SegTable& tb, uint32_t x,
-                                             uint32_t head_pos, const RunCounts& c, int l,
-                                             const CSum* s, uint32_t* dbg_count,
-                                             uint32_t* dbg_kept, unsigned long long& n_touched,
-                                             unsigned long long& n_applied) {
-  if (l == 0) {
-    ++n_touched;
-    if (dbg_count) {
-      dbg_count[head_pos] = c.c_all;
-      dbg_kept[head_pos] = c.k_occ;
-    }
+// The message of table-local occurrence x in the offsets off[0..M] (any memory).
+__device__ __forceinline__ int message_of_any(const uint32_t* off, int M, uint32_t x) {
+  int lo = 0, hi = M;
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (off[mid] <= x)
+      lo = mid;
+    else
+      hi = mid;
   }
-  if (c.k_occ == 0u) return;  // every occurrence excluded: no step, tag unchanged
-  if (x >= (uint32_t)tb.rows) return;  // only after a latched consistency error
-  apply_slice<VEC, L, EPL>(tb, x, l, s, row_denominator(a.sparse_den, c.c_all, c.c_kept, a.M));
-  if (l == 0) {
-    tb.ver[x] = (int32_t)(a.k + 1);
-    ++n_applied;
+  return lo;
+}
+
+// One round's segment (a maximal run of equal keys inside the round).
+struct SegInfo {
+  uint32_t x;         // row
+  uint32_t head_pos;  // sorted position of its first occurrence in the round
+  uint32_t c_all, c_kept;
+  uint32_t kmask;     // kept positions of the round in this segment
+  uint32_t is_head;   // 1 if the row starts here, 0 if it continues from before
+};
+
+// Lane j copies gradient row j (d floats) into its staging slot: 16-byte
+// copies when d is a multiple of 4 (rows are then 16-byte aligned), else
+// 4-byte copies.
+__device__ __forceinline__ void stage_row(float* dst, const float* src, int d) {
+  if ((d & 3) == 0) {
+    for (int i = 0; i < d; i += 4)
+      asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst + i)),
+                   "l"(src + i)
+                   : "memory");
+  } else {
+    for (int i = 0; i < d; ++i)
+      asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst + i)),
+                   "l"(src + i)
+                   : "memory");
   }
 }
 
-template <int VEC, int L, int EPL>
+template <int EPL>
 __device__ __forceinline__ void write_record(const SegRecords& rec, int64_t wg, int slot, int d,
                                              uint32_t type, uint32_t x, uint32_t head_pos,
-                                             const RunCounts& c, int l, const CSum* s) {
-  const size_t base = ((size_t)wg * 2 + slot) * (size_t)d;
+                                             const RunCounts& c, int lane, int n_mine,
+                                             const CSum* acc) {
+  const size_t base = ((size_t)wg * 2 + slot) * (size_t)d + (size_t)lane * EPL;
 #pragma unroll
-  for (int e = 0; e < EPL; ++e) {
-#pragma unroll
-    for (int v = 0; v < VEC; ++v) {
-      const int idx = (e * L + l) * VEC + v;
-      if (idx < d) {
-        rec.hi[base + idx] = s[e * VEC + v].hi;
-        rec.lo[base + idx] = s[e * VEC + v].lo;
-      }
+  for (int e = 0; e < EPL; ++e)
+    if (e < n_mine) {
+      rec.hi[base + e] = acc[e].hi;
+      rec.lo[base + e] = acc[e].lo;
     }
-  }
-  if (l == 0) {
+  if (lane == 0) {
     uint32_t* m = rec.meta + ((size_t)wg * 2 + slot) * REC_META;
     m[1] = x;
     m[2] = c.c_all;
@@ -147,244 +163,284 @@ __device__ __forceinline__ void write_record(const SegRecords& rec, int64_t wg, 
   }
 }
 
-template <int VEC, int L, int EPL>
-__global__ void __launch_bounds__(SEG_THREADS)
+// A finished row: counters and debug record; if anything was kept, its
+// compensated sums go to the warp's queue with the row and the denominator.
+template <int EPL>
+__device__ __forceinline__ void enqueue_row(uint32_t x, uint32_t head_pos, const RunCounts& rc,
+                                            const StepArgs& a, int M, uint32_t v_t, int lane,
+                                            const CSum* acc, float* pend, uint32_t* pend_x,
+                                            float* pend_den, int& npend, uint32_t& n_touched,
+                                            uint32_t& n_applied, uint32_t* dbg_count,
+                                            uint32_t* dbg_kept) {
+  if (lane == 0) {
+    ++n_touched;
+    if (dbg_count) {
+      dbg_count[head_pos] = rc.c_all;
+      dbg_kept[head_pos] = rc.k_occ;
+    }
+  }
+  if (rc.k_occ == 0u || x >= v_t) return;  // nothing kept: no step, tag unchanged
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) pend[npend * 32 * EPL + lane * EPL + e] = csum_value(acc[e]);
+  if (lane == 0) {
+    pend_x[npend] = x;
+    pend_den[npend] = row_denominator(a.sparse_den, rc.c_all, rc.c_kept, M);
+    ++n_applied;
+  }
+  ++npend;
+}
+
+// Applies the queued rows, a batch at a time: all state loads of a batch
+// first, then the updates.
+template <int EPL, bool VECOK>
+__device__ __noinline__ void flush_rows(const StepArgs& a, const SegTable& tb, int lane, int e0,
+                                        int n_mine, bool active, const float* pend,
+                                        const uint32_t* pend_x, const float* pend_den,
+                                        int& npend) {
+  constexpr int PB = pb_rows<EPL>();
+  const int d = tb.d;
+  __syncwarp();
+  for (int b0 = 0; b0 < npend; b0 += PB) {
+    float w[PB][EPL], s0[PB][EPL], s1[PB][EPL];
+#pragma unroll
+    for (int i = 0; i < PB; ++i) {
+      if (b0 + i < npend && active) {
+        const size_t rb = (size_t)pend_x[b0 + i] * (size_t)d + e0;
+        load_lane<EPL, VECOK>(tb.w + rb, n_mine, w[i]);
+        load_lane<EPL, VECOK>(tb.s0 + rb, n_mine, s0[i]);
+        if (tb.opt.kind == 1) load_lane<EPL, VECOK>(tb.s1 + rb, n_mine, s1[i]);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < PB; ++i) {
+      if (b0 + i < npend) {
+        const uint32_t x = pend_x[b0 + i];
+        if (active) {
+          const float den = pend_den[b0 + i];
+          const size_t rb = (size_t)x * (size_t)d + e0;
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) {
+            const float v = pend[(b0 + i) * 32 * EPL + lane * EPL + e];
+            opt_update(tb.opt, w[i][e], s0[i][e], s1[i][e], den == 1.0f ? v : __fdiv_rn(v, den));
+          }
+          store_lane<EPL, VECOK>(tb.w + rb, n_mine, w[i]);
+          store_lane<EPL, VECOK>(tb.s0 + rb, n_mine, s0[i]);
+          if (tb.opt.kind == 1) store_lane<EPL, VECOK>(tb.s1 + rb, n_mine, s1[i]);
+        }
+        if (lane == 0) tb.ver[x] = (int32_t)(a.k + 1);
+      }
+    }
+  }
+  npend = 0;
+  __syncwarp();
+}
+
+template <int EPL, bool VECOK>
+__global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 4 : (EPL == 2 ? 3 : 1))
     k_segsum_apply(StepArgs a, SegTable tb, const uint32_t* __restrict__ keys,
                    const uint32_t* __restrict__ vals, int64_t range, int64_t n_warps,
                    SegRecords rec, DevStats* st, uint32_t* dbg_count, uint32_t* dbg_kept,
                    ErrSink err) {
-  constexpr int G = 32 / L;  // lane groups per warp
-  constexpr int E = RS / G;  // positions per group slice
-  constexpr int NV = EPL * VEC;
-  __shared__ PosMeta s_meta[SEG_WARPS][RS];
+  constexpr int PB = pb_rows<EPL>();
+  constexpr int QR = queue_rows<EPL>();
+  constexpr int DS = 32 * EPL;  // staged row stride (floats)
+  __shared__ uint32_t s_off[MSG_CACHE + 1];
+  __shared__ int64_t s_tok[MSG_CACHE];
+  __shared__ const float* s_rowp[MSG_CACHE];
+  __shared__ SegInfo s_seg[SEG_WARPS][RS];
+  __shared__ uint32_t s_pend_x[SEG_WARPS][QR];
+  __shared__ float s_pend_den[SEG_WARPS][QR];
+  extern __shared__ __align__(16) float s_dyn[];  // staged rows, then the queue
 
   if (ld_volatile_u32(err.dev) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  const int M = a.M;
+  const uint32_t* off_g = a.msg_off + (size_t)tb.t * (M + 1);
+  const float* const* rows_g = a.rows_ptr + (size_t)tb.t * M;
+  const bool cached = M <= MSG_CACHE;
+  if (cached) {
+    for (int i = threadIdx.x; i <= M; i += SEG_THREADS) s_off[i] = off_g[i];
+    for (int i = threadIdx.x; i < M; i += SEG_THREADS) {
+      s_tok[i] = a.tokens[i];
+      s_rowp[i] = rows_g[i];
+    }
+  }
+  __syncthreads();
+  const uint32_t* off = cached ? s_off : off_g;
+
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t wg = (int64_t)blockIdx.x * SEG_WARPS + warp;
   if (wg >= n_warps) return;
-  const int g = lane / L, l = lane % L;
   const int d = tb.d;
-  const int M = a.M;
+  const int e0 = lane * EPL;  // first row element of this lane
+  const int n_mine = d - e0 < 0 ? 0 : (d - e0 < EPL ? d - e0 : EPL);
+  const bool active = n_mine > 0;
   const int64_t r0 = tb.pos_begin + wg * range;
   const int64_t r1 = (r0 + range < tb.pos_end) ? r0 + range : tb.pos_end;
-  const uint32_t* off = a.msg_off + (size_t)tb.t * (M + 1);
-  const float* const* rows_ptr = a.rows_ptr + (size_t)tb.t * M;
   const int64_t nbase = a.nbase[tb.t];
   const uint32_t n_t = (uint32_t)(tb.pos_end - tb.pos_begin);
   const uint32_t v_t = (uint32_t)tb.rows;
+  const uint32_t lt_mask = (1u << lane) - 1u;
 
-  unsigned long long n_pairs = 0, n_pairs_dropped = 0, stale_sum = 0, stale_max = 0;
-  unsigned long long n_touched = 0, n_applied = 0, n_kept_occ = 0;
+  uint32_t n_pairs = 0, n_pairs_dropped = 0, n_touched = 0, n_applied = 0, n_kept_occ = 0;
+  unsigned long long stale_sum = 0, stale_max = 0;
 
-  PosMeta* sm = s_meta[warp];
+  float* stage = s_dyn + (size_t)warp * RS * DS;
+  float* pend = s_dyn + (size_t)SEG_WARPS * RS * DS + (size_t)warp * QR * DS;
+  uint32_t* pend_x = s_pend_x[warp];
+  float* pend_den = s_pend_den[warp];
+  SegInfo* seg = s_seg[warp];
+  int npend = 0;
 
-  // State carried between positions: the key and message of the previous one.
+  // The row (run) open at the current position; the whole warp holds it,
+  // lane l its elements [l*EPL, (l+1)*EPL).
+  CSum acc[EPL];
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) acc[e] = CSum{0.f, 0.f};
+  RunCounts rc{0u, 0u, 0u};
+  uint32_t run_x = 0u, run_head = 0u;
+  bool run_active = false, run_local = false;
+  bool wrote_head_record = false, wrote_tail_record = false;
+
   uint32_t prev_key = 0xFFFFFFFFu, prev_m = 0xFFFFFFFFu;
   if (r0 > tb.pos_begin && r0 < r1) {
     prev_key = keys[r0 - 1];
-    prev_m = (uint32_t)message_of(off, M, (uint32_t)((int64_t)vals[r0 - 1] - nbase));
+    const uint32_t o_t = (uint32_t)((int64_t)vals[r0 - 1] - nbase);
+    prev_m = o_t < n_t ? (uint32_t)message_of_any(off, M, o_t) : 0xFFFFFFFFu;
+    if (prev_key == keys[r0]) {  // the range begins inside a row owned by an earlier range
+      run_active = true;
+      run_x = keys[r0] - tb.key_base;
+    }
   }
-
-  // The run open at the current boundary, replicated across groups.
-  CSum carry[NV];
-#pragma unroll
-  for (int i = 0; i < NV; ++i) carry[i] = CSum{0.f, 0.f};
-  RunCounts cc{0u, 0u, 0u};
-  uint32_t carry_x = 0u, carry_head = 0u;
-  bool carry_active = false, carry_local = false;
-  if (r0 < r1 && prev_key == keys[r0]) {  // range starts inside a row owned by an earlier warp
-    carry_active = true;
-    carry_x = keys[r0] - tb.key_base;
-  }
-  bool wrote_head_record = false, wrote_tail_record = false;
 
   for (int64_t rb = r0; rb < r1; rb += RS) {
     const int n_round = (int)((r1 - rb) < RS ? (r1 - rb) : RS);
-    // ---- per-position metadata (two positions per lane)
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int j = q * 32 + lane;
-      if (j < n_round) {
-        const uint32_t key = keys[rb + j];
-        const uint32_t o_t = (uint32_t)((int64_t)vals[rb + j] - nbase);
-        const uint32_t x = key - tb.key_base;
-        if (o_t >= n_t || x >= v_t) {
-          // cannot happen for a correctly sorted array; never touch memory with it
-          raise_error(err, ERR_INTERNAL);
-          sm[j].row = nullptr;
-          sm[j].key = key;
-          sm[j].m = 0u;
-          sm[j].pad = 0u;
-          sm[j].flags = 0u;
-          continue;
-        }
-        const int m = message_of(off, M, o_t);
-        const uint32_t p = o_t - __ldg(off + m);
+    const bool valid = lane < n_round;
+    // ---- lane j: metadata of position rb + j; stage its gradient row if kept
+    uint32_t key = 0xFFFFFFFFu, m = 0xFFFFFFFEu, stale = 0u;
+    bool keep = false;
+    if (valid) {
+      key = keys[rb + lane];
+      const uint32_t o_t = (uint32_t)((int64_t)vals[rb + lane] - nbase);
+      const uint32_t x = key - tb.key_base;
+      if (o_t >= n_t || x >= v_t) {
+        // cannot happen for a correctly sorted array; never touch memory with it
+        raise_error(err, ERR_INTERNAL);
+      } else {
+        m = (uint32_t)message_of_any(off, M, o_t);
+        const uint32_t p = o_t - off[m];
+        const int64_t tok = cached ? s_tok[m] : a.tokens[m];
+        const float* rowp = (cached ? s_rowp[m] : rows_g[m]) + (size_t)p * (size_t)d;
         const int64_t ref = a.row_staleness == 0 ? (int64_t)tb.ver[x] : a.k;
-        const int64_t diff = ref - a.tokens[m];
-        const uint64_t s = diff > 0 ? (uint64_t)diff : 0ull;
-        const bool keep = s <= (uint64_t)(int64_t)a.iota;
-        sm[j].row = rows_ptr[m] + (size_t)p * (size_t)d;
-        sm[j].key = key;
-        sm[j].m = (uint32_t)m;
-        sm[j].pad = (uint32_t)(s > 0xFFFFFFFFull ? 0xFFFFFFFFull : s);
-        sm[j].flags = keep ? F_KEEP : 0u;
+        const int64_t diff = ref - tok;
+        const uint64_t sl = diff > 0 ? (uint64_t)diff : 0ull;
+        keep = sl <= (uint64_t)(int64_t)a.iota;
+        stale = (uint32_t)(sl > 0xFFFFFFFFull ? 0xFFFFFFFFull : sl);
+        if (keep) stage_row(stage + lane * DS, rowp, d);
       }
     }
-    __syncwarp();
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      const int j = q * 32 + lane;
-      if (j < n_round) {
-        const uint32_t pk = j == 0 ? prev_key : sm[j - 1].key;
-        const uint32_t pm = j == 0 ? prev_m : sm[j - 1].m;
-        if (sm[j].flags & F_KEEP) ++n_kept_occ;
-        const bool head = sm[j].key != pk;
-        const bool newmsg = head || sm[j].m != pm;
-        uint32_t f = sm[j].flags;
-        if (head) f |= F_HEAD;
-        if (newmsg) {
-          f |= F_NEWMSG;
-          ++n_pairs;
-          if (!(f & F_KEEP)) ++n_pairs_dropped;
-          const unsigned long long s = sm[j].pad;
-          stale_sum += s;
-          stale_max = s > stale_max ? s : stale_max;
-        }
-        sm[j].flags = f;  // written after all reads of this round's neighbours below
-      }
+    uint32_t pk = __shfl_up_sync(0xffffffffu, key, 1);
+    uint32_t pm = __shfl_up_sync(0xffffffffu, m, 1);
+    if (lane == 0) {
+      pk = prev_key;
+      pm = prev_m;
     }
+    const bool head = valid && key != pk;
+    const bool newmsg = valid && (head || m != pm);
+    if (keep) ++n_kept_occ;
+    if (newmsg) {
+      ++n_pairs;
+      if (!keep) ++n_pairs_dropped;
+      stale_sum += stale;
+      stale_max = stale > stale_max ? stale : stale_max;
+    }
+    const uint32_t Hm = __ballot_sync(0xffffffffu, head);
+    const uint32_t Km = __ballot_sync(0xffffffffu, keep);
+    const uint32_t Nm = __ballot_sync(0xffffffffu, newmsg);
+    const uint32_t Vm = __ballot_sync(0xffffffffu, valid);
+    // ---- segments of the round (position 0 always starts one): lane-parallel
+    const uint32_t Bm = (Hm | 1u) & Vm;
+    if ((Bm >> lane) & 1u) {
+      const uint32_t above = lane == 31 ? 0u : (Bm & ~((2u << lane) - 1u));
+      const int end = above ? __ffs(above) - 1 : n_round;
+      const uint32_t rng = (end >= 32 ? 0xFFFFFFFFu : ((1u << end) - 1u)) & ~lt_mask;
+      SegInfo& sg = seg[__popc(Bm & lt_mask)];
+      sg.x = key - tb.key_base;
+      sg.head_pos = (uint32_t)(rb + lane);
+      sg.c_all = __popc(Nm & rng);
+      sg.c_kept = __popc(Nm & Km & rng);
+      sg.kmask = Km & rng;
+      sg.is_head = head ? 1u : 0u;
+    }
+    const int R = __popc(Bm);
+    prev_key = __shfl_sync(0xffffffffu, key, n_round - 1);
+    prev_m = __shfl_sync(0xffffffffu, m, n_round - 1);
+    stage_wait_all();
     __syncwarp();
-    prev_key = sm[n_round - 1].key;
-    prev_m = sm[n_round - 1].m;
 
-    // ---- each group walks its slice sequentially
-    const int j0 = g * E;
-    CSum acc[NV], cont[NV];
-#pragma unroll
-    for (int i = 0; i < NV; ++i) acc[i] = cont[i] = CSum{0.f, 0.f};
-    RunCounts ac{0u, 0u, 0u}, cn{0u, 0u, 0u};
-    uint32_t a_x = 0u, a_head = 0u;
-    bool in_cont = (j0 < n_round) && !(sm[j0].flags & F_HEAD);
-    bool have_open = false;
-    bool any_head = false;
-#pragma unroll 4
-    for (int jj = 0; jj < E; ++jj) {
-      const int j = j0 + jj;
-      if (j < n_round) {
-        const uint32_t f = sm[j].flags;
-        if (f & F_HEAD) {
-          any_head = true;
-          if (in_cont) {  // the row continued from before ends here
-#pragma unroll
-            for (int i = 0; i < NV; ++i) cont[i] = acc[i];
-            cn = ac;
-            in_cont = false;
-          } else if (have_open) {  // a row that started in this slice is complete
-            finalize_row<VEC, L, EPL>(a, tb, a_x, a_head, ac, l, acc, dbg_count, dbg_kept,
-                                      n_touched, n_applied);
-          }
-#pragma unroll
-          for (int i = 0; i < NV; ++i) acc[i] = CSum{0.f, 0.f};
-          ac = RunCounts{0u, 0u, 0u};
-          a_x = sm[j].key - tb.key_base;
-          a_head = (uint32_t)(rb + j);
-          have_open = true;
-        }
-        if (f & F_NEWMSG) {
-          ++ac.c_all;
-          if (f & F_KEEP) ++ac.c_kept;
-        }
-        if (f & F_KEEP) {
-          ++ac.k_occ;
-          const float* row = sm[j].row;
-#pragma unroll
-          for (int e = 0; e < EPL; ++e) {
-            const int idx = (e * L + l) * VEC;
-            if (idx < d) {
-              float v[VEC];
-              Vec<VEC>::load(row + idx, v);
-#pragma unroll
-              for (int u = 0; u < VEC; ++u) csum_add(acc[e * VEC + u], v[u]);
-            }
+    // ---- walk the round segment by segment (uniform control flow)
+    for (int r = 0; r < R; ++r) {
+      const SegInfo sg = seg[r];
+      if (sg.is_head) {
+        if (run_active) {
+          // finish the open row: queue its aggregated gradient (or, for a row
+          // that began in an earlier range, leave the partial for the fixup)
+          if (!run_local) {
+            write_record<EPL>(rec, wg, 0, d, REC_CLOSED, run_x, 0u, rc, lane, n_mine, acc);
+            wrote_head_record = true;
+          } else {
+            enqueue_row<EPL>(run_x, run_head, rc, a, M, v_t, lane, acc, pend, pend_x, pend_den,
+                             npend, n_touched, n_applied, dbg_count, dbg_kept);
+            if (npend >= PB)
+              flush_rows<EPL, VECOK>(a, tb, lane, e0, n_mine, active, pend, pend_x, pend_den,
+                                     npend);
           }
         }
-      }
-    }
-    // acc: the open run (started at a head in the slice) or, with no head in the
-    // slice, the part of the continued row (pass-through).
-    const uint32_t head_mask = __ballot_sync(0xffffffffu, any_head && l == 0);
-
-    // ---- stitch the slices of this round in order
-    for (int gg = 0; gg < G; ++gg) {
-      if (gg * E >= n_round) break;
-      const int src = gg * L + l;
-      const bool starts_head = (sm[gg * E].flags & F_HEAD) != 0u;
-      const bool has_head = (head_mask >> (gg * L)) & 1u;
-      if (!starts_head) {
-        // continuation of the carried row: its part in slice gg is `cont` if a
-        // head closes it inside the slice, else the whole slice (`acc`).
 #pragma unroll
-        for (int i = 0; i < NV; ++i) {
-          const float hi = __shfl_sync(0xffffffffu, has_head ? cont[i].hi : acc[i].hi, src);
-          const float lo = __shfl_sync(0xffffffffu, has_head ? cont[i].lo : acc[i].lo, src);
-          csum_merge(carry[i], hi, lo);
-        }
-        cc.c_all += __shfl_sync(0xffffffffu, has_head ? cn.c_all : ac.c_all, gg * L);
-        cc.c_kept += __shfl_sync(0xffffffffu, has_head ? cn.c_kept : ac.c_kept, gg * L);
-        cc.k_occ += __shfl_sync(0xffffffffu, has_head ? cn.k_occ : ac.k_occ, gg * L);
-        if (!has_head) continue;  // the row continues past this slice
+        for (int e = 0; e < EPL; ++e) acc[e] = CSum{0.f, 0.f};
+        rc = RunCounts{sg.c_all, sg.c_kept, (uint32_t)__popc(sg.kmask)};
+        run_x = sg.x;
+        run_head = sg.head_pos;
+        run_active = true;
+        run_local = true;
+      } else {
+        rc.c_all += sg.c_all;
+        rc.c_kept += sg.c_kept;
+        rc.k_occ += __popc(sg.kmask);
       }
-      // The carried row (if any) is complete here.
-      if (carry_active) {
-        if (carry_local) {
-          if (g == 0)
-            finalize_row<VEC, L, EPL>(a, tb, carry_x, carry_head, cc, l, carry, dbg_count,
-                                      dbg_kept, n_touched, n_applied);
-        } else {
-          if (g == 0)
-            write_record<VEC, L, EPL>(rec, wg, 0, d, REC_CLOSED, carry_x, 0u, cc, l, carry);
-          wrote_head_record = true;
-        }
-      }
-      // The open run of slice gg becomes the carried row.
+      uint32_t km = sg.kmask;
+      while (km) {
+        const int j = __ffs(km) - 1;
+        km &= km - 1u;
+        float v[EPL];
+        load_lane<EPL, true>(stage + j * DS + e0, EPL, v);
 #pragma unroll
-      for (int i = 0; i < NV; ++i) {
-        carry[i].hi = __shfl_sync(0xffffffffu, acc[i].hi, src);
-        carry[i].lo = __shfl_sync(0xffffffffu, acc[i].lo, src);
+        for (int e = 0; e < EPL; ++e) csum_add(acc[e], v[e]);
       }
-      cc.c_all = __shfl_sync(0xffffffffu, ac.c_all, gg * L);
-      cc.c_kept = __shfl_sync(0xffffffffu, ac.c_kept, gg * L);
-      cc.k_occ = __shfl_sync(0xffffffffu, ac.k_occ, gg * L);
-      carry_x = __shfl_sync(0xffffffffu, a_x, gg * L);
-      carry_head = __shfl_sync(0xffffffffu, a_head, gg * L);
-      carry_active = true;
-      carry_local = true;
     }
     __syncwarp();
   }
 
-  // ---- end of the range: the carried row ends here or continues in the next range
-  if (carry_active) {
+  // ---- end of the range: the open row ends here or continues in the next range
+  if (run_active) {
     const bool closes = (r1 == tb.pos_end) || keys[r1] != keys[r1 - 1];
     if (closes) {
-      if (carry_local) {
-        if (g == 0)
-          finalize_row<VEC, L, EPL>(a, tb, carry_x, carry_head, cc, l, carry, dbg_count,
-                                    dbg_kept, n_touched, n_applied);
-      } else {
-        if (g == 0) write_record<VEC, L, EPL>(rec, wg, 0, d, REC_CLOSED, carry_x, 0u, cc, l, carry);
+      if (!run_local) {
+        write_record<EPL>(rec, wg, 0, d, REC_CLOSED, run_x, 0u, rc, lane, n_mine, acc);
         wrote_head_record = true;
+      } else {
+        enqueue_row<EPL>(run_x, run_head, rc, a, M, v_t, lane, acc, pend, pend_x, pend_den,
+                         npend, n_touched, n_applied, dbg_count, dbg_kept);
       }
-    } else if (carry_local) {
-      if (g == 0)
-        write_record<VEC, L, EPL>(rec, wg, 1, d, REC_OWNER, carry_x, carry_head, cc, l, carry);
+    } else if (run_local) {
+      write_record<EPL>(rec, wg, 1, d, REC_OWNER, run_x, run_head, rc, lane, n_mine, acc);
       wrote_tail_record = true;
     } else {
-      if (g == 0) write_record<VEC, L, EPL>(rec, wg, 0, d, REC_PASS, carry_x, 0u, cc, l, carry);
+      write_record<EPL>(rec, wg, 0, d, REC_PASS, run_x, 0u, rc, lane, n_mine, acc);
       wrote_head_record = true;
     }
   }
+  if (npend > 0)
+    flush_rows<EPL, VECOK>(a, tb, lane, e0, n_mine, active, pend, pend_x, pend_den, npend);
   if (lane == 0) {
     if (!wrote_head_record) rec.meta[((size_t)wg * 2 + 0) * REC_META] = REC_NONE;
     if (!wrote_tail_record) rec.meta[((size_t)wg * 2 + 1) * REC_META] = REC_NONE;
@@ -398,18 +454,383 @@ __global__ void __launch_bounds__(SEG_THREADS)
     stale_sum += __shfl_xor_sync(0xffffffffu, stale_sum, o);
     const unsigned long long y = __shfl_xor_sync(0xffffffffu, stale_max, o);
     stale_max = y > stale_max ? y : stale_max;
-    n_touched += __shfl_xor_sync(0xffffffffu, n_touched, o);
-    n_applied += __shfl_xor_sync(0xffffffffu, n_applied, o);
     n_kept_occ += __shfl_xor_sync(0xffffffffu, n_kept_occ, o);
   }
   if (lane == 0) {
-    if (n_pairs) atomicAdd(&st->pairs, n_pairs);
-    if (n_pairs_dropped) atomicAdd(&st->pairs_dropped, n_pairs_dropped);
+    if (n_pairs) atomicAdd(&st->pairs, (unsigned long long)n_pairs);
+    if (n_pairs_dropped) atomicAdd(&st->pairs_dropped, (unsigned long long)n_pairs_dropped);
     if (stale_sum) atomicAdd(&st->row_stale_sum, stale_sum);
     if (stale_max) atomicMax(&st->row_stale_max, stale_max);
-    if (n_touched) atomicAdd(&st->rows_touched, n_touched);
-    if (n_applied) atomicAdd(&st->rows_applied, n_applied);
-    if (n_kept_occ) atomicAdd(&st->occ_kept, n_kept_occ);
+    if (n_touched) atomicAdd(&st->rows_touched, (unsigned long long)n_touched);
+    if (n_applied) atomicAdd(&st->rows_applied, (unsigned long long)n_applied);
+    if (n_kept_occ) atomicAdd(&st->occ_kept, (unsigned long long)n_kept_occ);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Rows of up to 64 floats: most unique rows of a round occur once, so they are
+// handled lane-parallel, and the optimizer runs with one lane per row.
+//
+// Per round of 32 positions: lane j computes position j's metadata and stages
+// its gradient row in shared memory; the round's segments (maximal runs of
+// equal keys) are found with ballots.  A segment that starts and ends inside
+// the round with at most one kept occurrence is queued by its own lane (its
+// row copied, no arithmetic).  The first segment (which may continue the row
+// open from the previous round), segments with several kept occurrences, and
+// the last segment (which may continue into the next round) are summed by the
+// whole warp, lane = element, with compensated arithmetic.  Queued rows are
+// applied with lane = row: each lane streams its row's gradient, weights and
+// optimizer state in 16-byte pieces.
+// ---------------------------------------------------------------------------
+constexpr int QCAP = 64;  // queued rows per warp
+
+template <int EPL>
+__host__ __device__ constexpr int row_stride() { return 32 * EPL + 4; }  // floats, bank-skewed
+template <int EPL>
+__host__ __device__ constexpr size_t rows_dyn_smem() {
+  return (size_t)SEG_WARPS * (RS + QCAP) * row_stride<EPL>() * sizeof(float);
+}
+
+__device__ __forceinline__ void copy_row_smem(float* dst, const float* src, int d) {
+  if ((d & 3) == 0) {
+    for (int i = 0; i < d; i += 4)
+      *reinterpret_cast<float4*>(dst + i) = *reinterpret_cast<const float4*>(src + i);
+  } else {
+    for (int i = 0; i < d; ++i) dst[i] = src[i];
+  }
+}
+
+// Lane = row: applies queued rows [0, npend), 32 at a time.
+__device__ __noinline__ void apply_queue(const StepArgs& a, const SegTable& tb, int lane,
+                                         const float* pend, const uint32_t* pend_x,
+                                         const float* pend_den, int qs, int& npend) {
+  const int d = tb.d;
+  const bool adam = tb.opt.kind == 1;
+  __syncwarp();
+  for (int b0 = 0; b0 < npend; b0 += 32) {
+    const int i = b0 + lane;
+    if (i < npend) {
+      const uint32_t x = pend_x[i];
+      const float den = pend_den[i];
+      const float* g = pend + (size_t)i * qs;
+      float* w = tb.w + (size_t)x * d;
+      float* s0 = tb.s0 + (size_t)x * d;
+      float* s1 = adam ? tb.s1 + (size_t)x * d : nullptr;
+      if ((d & 3) == 0) {
+        constexpr int U = 2;  // 16-byte pieces in flight per lane and array
+        for (int c0 = 0; c0 < d; c0 += 4 * U) {
+          float4 wv[U], av[U], bv[U], gv[U];
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int c = c0 + 4 * u;
+            if (c < d) {
+              wv[u] = *reinterpret_cast<const float4*>(w + c);
+              av[u] = *reinterpret_cast<const float4*>(s0 + c);
+              if (adam) bv[u] = *reinterpret_cast<const float4*>(s1 + c);
+              gv[u] = *reinterpret_cast<const float4*>(g + c);
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int c = c0 + 4 * u;
+            if (c < d) {
+              float* wp = &wv[u].x;
+              float* ap = &av[u].x;
+              float* bp = &bv[u].x;
+              const float* gp = &gv[u].x;
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                float bk = adam ? bp[k] : 0.f;
+                opt_update(tb.opt, wp[k], ap[k], bk, den == 1.0f ? gp[k] : __fdiv_rn(gp[k], den));
+                bp[k] = bk;
+              }
+              *reinterpret_cast<float4*>(w + c) = wv[u];
+              *reinterpret_cast<float4*>(s0 + c) = av[u];
+              if (adam) *reinterpret_cast<float4*>(s1 + c) = bv[u];
+            }
+          }
+        }
+      } else {
+        for (int c = 0; c < d; ++c) {
+          float wk = w[c], ak = s0[c], bk = adam ? s1[c] : 0.f;
+          opt_update(tb.opt, wk, ak, bk, den == 1.0f ? g[c] : __fdiv_rn(g[c], den));
+          w[c] = wk;
+          s0[c] = ak;
+          if (adam) s1[c] = bk;
+        }
+      }
+      tb.ver[x] = (int32_t)(a.k + 1);
+    }
+  }
+  npend = 0;
+  __syncwarp();
+}
+
+template <int EPL>
+__global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 3 : 2)
+    k_segsum_rows(StepArgs a, SegTable tb, const uint32_t* __restrict__ keys,
+                  const uint32_t* __restrict__ vals, int64_t range, int64_t n_warps,
+                  SegRecords rec, DevStats* st, uint32_t* dbg_count, uint32_t* dbg_kept,
+                  ErrSink err) {
+  constexpr int SS = row_stride<EPL>();
+  __shared__ uint32_t s_off[MSG_CACHE + 1];
+  __shared__ int64_t s_tok[MSG_CACHE];
+  __shared__ const float* s_rowp[MSG_CACHE];
+  __shared__ uint4 s_seg[SEG_WARPS][RS];  // by start position: x, head_pos, kmask, counts
+  __shared__ uint32_t s_pend_x[SEG_WARPS][QCAP];
+  __shared__ float s_pend_den[SEG_WARPS][QCAP];
+  extern __shared__ __align__(16) float s_dyn[];  // staged rows, then the queue
+
+  if (ld_volatile_u32(err.dev) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  const int M = a.M;
+  const uint32_t* off_g = a.msg_off + (size_t)tb.t * (M + 1);
+  const float* const* rows_g = a.rows_ptr + (size_t)tb.t * M;
+  const bool cached = M <= MSG_CACHE;
+  if (cached) {
+    for (int i = threadIdx.x; i <= M; i += SEG_THREADS) s_off[i] = off_g[i];
+    for (int i = threadIdx.x; i < M; i += SEG_THREADS) {
+      s_tok[i] = a.tokens[i];
+      s_rowp[i] = rows_g[i];
+    }
+  }
+  __syncthreads();
+  const uint32_t* off = cached ? s_off : off_g;
+
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t wg = (int64_t)blockIdx.x * SEG_WARPS + warp;
+  if (wg >= n_warps) return;
+  const int d = tb.d;
+  const int qs = ((d + 3) & ~3) + 4;  // queued row stride
+  const int e0 = lane * EPL;
+  const int n_mine = d - e0 < 0 ? 0 : (d - e0 < EPL ? d - e0 : EPL);
+  const int64_t r0 = tb.pos_begin + wg * range;
+  const int64_t r1 = (r0 + range < tb.pos_end) ? r0 + range : tb.pos_end;
+  const int64_t nbase = a.nbase[tb.t];
+  const uint32_t n_t = (uint32_t)(tb.pos_end - tb.pos_begin);
+  const uint32_t v_t = (uint32_t)tb.rows;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  const int mode = a.sparse_den;
+
+  uint32_t n_pairs = 0, n_pairs_dropped = 0, n_touched = 0, n_applied = 0, n_kept_occ = 0;
+  unsigned long long stale_sum = 0, stale_max = 0;
+
+  float* stage = s_dyn + (size_t)warp * RS * SS;
+  float* pend = s_dyn + (size_t)SEG_WARPS * RS * SS + (size_t)warp * QCAP * SS;
+  uint32_t* pend_x = s_pend_x[warp];
+  float* pend_den = s_pend_den[warp];
+  uint4* seg = s_seg[warp];
+  int npend = 0;
+
+  CSum acc[EPL];
+#pragma unroll
+  for (int e = 0; e < EPL; ++e) acc[e] = CSum{0.f, 0.f};
+  RunCounts rc{0u, 0u, 0u};
+  uint32_t run_x = 0u, run_head = 0u;
+  bool run_active = false, run_local = false;
+  bool wrote_head_record = false, wrote_tail_record = false;
+
+  uint32_t prev_key = 0xFFFFFFFFu, prev_m = 0xFFFFFFFFu;
+  if (r0 > tb.pos_begin && r0 < r1) {
+    prev_key = keys[r0 - 1];
+    const uint32_t o_t = (uint32_t)((int64_t)vals[r0 - 1] - nbase);
+    prev_m = o_t < n_t ? (uint32_t)message_of_any(off, M, o_t) : 0xFFFFFFFFu;
+    if (prev_key == keys[r0]) {  // the range begins inside a row owned by an earlier range
+      run_active = true;
+      run_x = keys[r0] - tb.key_base;
+    }
+  }
+
+  // the warp-held row is complete: queue it (or hand it to the fixup kernel)
+  auto finish_run = [&]() {
+    if (!run_local) {
+      write_record<EPL>(rec, wg, 0, d, REC_CLOSED, run_x, 0u, rc, lane, n_mine, acc);
+      wrote_head_record = true;
+      return;
+    }
+    if (lane == 0) {
+      ++n_touched;
+      if (dbg_count) {
+        dbg_count[run_head] = rc.c_all;
+        dbg_kept[run_head] = rc.k_occ;
+      }
+    }
+    if (rc.k_occ == 0u || run_x >= v_t) return;
+#pragma unroll
+    for (int e = 0; e < EPL; ++e)
+      if (e < n_mine) pend[npend * qs + e0 + e] = csum_value(acc[e]);
+    if (lane == 0) {
+      pend_x[npend] = run_x;
+      pend_den[npend] = row_denominator(mode, rc.c_all, rc.c_kept, M);
+      ++n_applied;
+    }
+    ++npend;
+  };
+
+  for (int64_t rb = r0; rb < r1; rb += RS) {
+    const int n_round = (int)((r1 - rb) < RS ? (r1 - rb) : RS);
+    const bool valid = lane < n_round;
+    // ---- lane j: metadata of position rb + j; its gradient row is staged if kept
+    uint32_t key = 0xFFFFFFFFu, m = 0xFFFFFFFEu, stale = 0u;
+    bool keep = false;
+    if (valid) {
+      key = keys[rb + lane];
+      const uint32_t o_t = (uint32_t)((int64_t)vals[rb + lane] - nbase);
+      const uint32_t x = key - tb.key_base;
+      if (o_t >= n_t || x >= v_t) {
+        raise_error(err, ERR_INTERNAL);  // cannot happen for a correctly sorted array
+      } else {
+        m = (uint32_t)message_of_any(off, M, o_t);
+        const uint32_t p = o_t - off[m];
+        const int64_t tok = cached ? s_tok[m] : a.tokens[m];
+        const float* rowp = (cached ? s_rowp[m] : rows_g[m]) + (size_t)p * (size_t)d;
+        const int64_t ref = a.row_staleness == 0 ? (int64_t)tb.ver[x] : a.k;
+        const int64_t diff = ref - tok;
+        const uint64_t sl = diff > 0 ? (uint64_t)diff : 0ull;
+        keep = sl <= (uint64_t)(int64_t)a.iota;
+        stale = (uint32_t)(sl > 0xFFFFFFFFull ? 0xFFFFFFFFull : sl);
+        if (keep) stage_row(stage + lane * SS, rowp, d);
+      }
+    }
+    uint32_t pk = __shfl_up_sync(0xffffffffu, key, 1);
+    uint32_t pm = __shfl_up_sync(0xffffffffu, m, 1);
+    if (lane == 0) {
+      pk = prev_key;
+      pm = prev_m;
+    }
+    const bool head = valid && key != pk;
+    const bool newmsg = valid && (head || m != pm);
+    if (keep) ++n_kept_occ;
+    if (newmsg) {
+      ++n_pairs;
+      if (!keep) ++n_pairs_dropped;
+      stale_sum += stale;
+      stale_max = stale > stale_max ? stale : stale_max;
+    }
+    const uint32_t Hm = __ballot_sync(0xffffffffu, head);
+    const uint32_t Km = __ballot_sync(0xffffffffu, keep);
+    const uint32_t Nm = __ballot_sync(0xffffffffu, newmsg);
+    const uint32_t Vm = __ballot_sync(0xffffffffu, valid);
+    const uint32_t Bm = (Hm | 1u) & Vm;  // segment starts (position 0 always starts one)
+    const int last_start = 31 - __clz(Bm);
+    const bool starts = (Bm >> lane) & 1u;
+    bool single = false, single_apply = false;
+    uint32_t kmask = 0u, c_all = 0u, c_kept = 0u;
+    if (starts) {
+      const uint32_t above = lane == 31 ? 0u : (Bm & ~((2u << lane) - 1u));
+      const int end = above ? __ffs(above) - 1 : n_round;
+      const uint32_t rng = (end >= 32 ? 0xFFFFFFFFu : ((1u << end) - 1u)) & ~lt_mask;
+      kmask = Km & rng;
+      c_all = __popc(Nm & rng);
+      c_kept = __popc(Nm & Km & rng);
+      single = lane > 0 && lane < last_start && __popc(kmask) <= 1;
+      single_apply = single && kmask != 0u;
+      seg[lane] = make_uint4(key - tb.key_base, (uint32_t)(rb + lane), kmask,
+                             c_all | (c_kept << 8) | (head ? 1u << 16 : 0u));
+    }
+    const uint32_t Sm = __ballot_sync(0xffffffffu, single_apply);
+    const uint32_t Um = Bm & ~__ballot_sync(0xffffffffu, single);
+    prev_key = __shfl_sync(0xffffffffu, key, n_round - 1);
+    prev_m = __shfl_sync(0xffffffffu, m, n_round - 1);
+    stage_wait_all();
+    __syncwarp();
+    // a round queues at most one row per segment plus the row it closes
+    if (npend > QCAP - 33) apply_queue(a, tb, lane, pend, pend_x, pend_den, qs, npend);
+
+    // ---- rows that occur once in the round, inside it: their own lane queues them
+    if (single) {
+      ++n_touched;
+      if (dbg_count) {
+        dbg_count[rb + lane] = c_all;
+        dbg_kept[rb + lane] = __popc(kmask);
+      }
+      if (single_apply) {
+        const int slot = npend + __popc(Sm & lt_mask);
+        const int pj = __ffs(kmask) - 1;
+        copy_row_smem(pend + slot * qs, stage + pj * SS, d);
+        pend_x[slot] = key - tb.key_base;
+        pend_den[slot] = row_denominator(mode, c_all, c_kept, M);
+        ++n_applied;
+      }
+    }
+    npend += __popc(Sm);
+
+    // ---- the other segments, in order, summed by the whole warp
+    uint32_t um = Um;
+    while (um) {
+      const int j = __ffs(um) - 1;
+      um &= um - 1u;
+      const uint4 sg = seg[j];
+      const bool is_head = (sg.w >> 16) & 1u;
+      const uint32_t s_call = sg.w & 0xFFu, s_ckept = (sg.w >> 8) & 0xFFu;
+      if (!is_head) {  // continues the open row (only at j == 0)
+        rc.c_all += s_call;
+        rc.c_kept += s_ckept;
+        rc.k_occ += __popc(sg.z);
+      } else {
+        if (run_active) finish_run();  // the open row ended before this head
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) acc[e] = CSum{0.f, 0.f};
+        rc = RunCounts{s_call, s_ckept, (uint32_t)__popc(sg.z)};
+        run_x = sg.x;
+        run_head = sg.y;
+        run_active = true;
+        run_local = true;
+      }
+      uint32_t km = sg.z;
+      while (km) {
+        const int pj = __ffs(km) - 1;
+        km &= km - 1u;
+        float v[EPL];
+        load_lane<EPL, true>(stage + pj * SS + e0, EPL, v);
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) csum_add(acc[e], v[e]);
+      }
+      // a segment before the round's last one ends inside the round
+      if (j < last_start) {
+        finish_run();
+        run_active = false;
+      }
+    }
+    __syncwarp();
+  }
+
+  // ---- end of the range: the open row ends here or continues in the next range
+  if (run_active) {
+    const bool closes = (r1 == tb.pos_end) || keys[r1] != keys[r1 - 1];
+    if (closes) {
+      finish_run();
+    } else if (run_local) {
+      write_record<EPL>(rec, wg, 1, d, REC_OWNER, run_x, run_head, rc, lane, n_mine, acc);
+      wrote_tail_record = true;
+    } else {
+      write_record<EPL>(rec, wg, 0, d, REC_PASS, run_x, 0u, rc, lane, n_mine, acc);
+      wrote_head_record = true;
+    }
+  }
+  if (npend > 0) apply_queue(a, tb, lane, pend, pend_x, pend_den, qs, npend);
+  if (lane == 0) {
+    if (!wrote_head_record) rec.meta[((size_t)wg * 2 + 0) * REC_META] = REC_NONE;
+    if (!wrote_tail_record) rec.meta[((size_t)wg * 2 + 1) * REC_META] = REC_NONE;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    n_pairs += __shfl_xor_sync(0xffffffffu, n_pairs, o);
+    n_pairs_dropped += __shfl_xor_sync(0xffffffffu, n_pairs_dropped, o);
+    stale_sum += __shfl_xor_sync(0xffffffffu, stale_sum, o);
+    const unsigned long long y = __shfl_xor_sync(0xffffffffu, stale_max, o);
+    stale_max = y > stale_max ? y : stale_max;
+    n_kept_occ += __shfl_xor_sync(0xffffffffu, n_kept_occ, o);
+    n_touched += __shfl_xor_sync(0xffffffffu, n_touched, o);
+    n_applied += __shfl_xor_sync(0xffffffffu, n_applied, o);
+  }
+  if (lane == 0) {
+    if (n_pairs) atomicAdd(&st->pairs, (unsigned long long)n_pairs);
+    if (n_pairs_dropped) atomicAdd(&st->pairs_dropped, (unsigned long long)n_pairs_dropped);
+    if (stale_sum) atomicAdd(&st->row_stale_sum, stale_sum);
+    if (stale_max) atomicMax(&st->row_stale_max, stale_max);
+    if (n_touched) atomicAdd(&st->rows_touched, (unsigned long long)n_touched);
+    if (n_applied) atomicAdd(&st->rows_applied, (unsigned long long)n_applied);
+    if (n_kept_occ) atomicAdd(&st->occ_kept, (unsigned long long)n_kept_occ);
   }
 }
 
@@ -444,28 +865,44 @@ __global__ void __launch_bounds__(256)
   }
   RunCounts c{m1[2], m1[3], m1[4]};
   const uint32_t head_pos = m1[5];
+  // Walk the following ranges in order; their record headers are read a window
+  // at a time (independent loads), then their partial sums are merged in order.
+  constexpr int FIX_WIN = 8;
   bool closed = false;
-  for (int64_t w2 = w + 1; w2 < n_warps; ++w2) {
-    const uint32_t* m0 = rec.meta + ((size_t)w2 * 2 + 0) * REC_META;
-    const uint32_t type = m0[0];
-    if ((type != REC_PASS && type != REC_CLOSED) || m0[1] != x) {
-      if (lane == 0) raise_error(err, ERR_INTERNAL);
-      return;
-    }
+  for (int64_t wb = w + 1; wb < n_warps && !closed; wb += FIX_WIN) {
+    uint32_t ty[FIX_WIN], rx[FIX_WIN];
 #pragma unroll
-    for (int i = 0; i < FIX_MAX_PER_LANE; ++i) {
-      const int idx = lane + 32 * i;
-      if (idx < d) {
-        const size_t b = ((size_t)w2 * 2 + 0) * d + idx;
-        csum_merge(s[i], rec.hi[b], rec.lo[b]);
+    for (int i = 0; i < FIX_WIN; ++i) {
+      const int64_t w2 = wb + i;
+      ty[i] = REC_NONE;
+      rx[i] = 0u;
+      if (w2 < n_warps) {
+        const uint32_t* m0 = rec.meta + ((size_t)w2 * 2 + 0) * REC_META;
+        ty[i] = m0[0];
+        rx[i] = m0[1];
       }
     }
-    c.c_all += m0[2];
-    c.c_kept += m0[3];
-    c.k_occ += m0[4];
-    if (type == REC_CLOSED) {
-      closed = true;
-      break;
+#pragma unroll
+    for (int i = 0; i < FIX_WIN; ++i) {
+      const int64_t w2 = wb + i;
+      if (closed || w2 >= n_warps) break;
+      if ((ty[i] != REC_PASS && ty[i] != REC_CLOSED) || rx[i] != x) {
+        if (lane == 0) raise_error(err, ERR_INTERNAL);
+        return;
+      }
+      const uint32_t* m0 = rec.meta + ((size_t)w2 * 2 + 0) * REC_META;
+#pragma unroll
+      for (int k = 0; k < FIX_MAX_PER_LANE; ++k) {
+        const int idx = lane + 32 * k;
+        if (idx < d) {
+          const size_t b = ((size_t)w2 * 2 + 0) * d + idx;
+          csum_merge(s[k], rec.hi[b], rec.lo[b]);
+        }
+      }
+      c.c_all += m0[2];
+      c.c_kept += m0[3];
+      c.k_occ += m0[4];
+      if (ty[i] == REC_CLOSED) closed = true;
     }
   }
   if (!closed) {
@@ -500,45 +937,92 @@ __global__ void __launch_bounds__(256)
   }
 }
 
-template <int VEC, int L, int EPL>
-void launch_cfg(const StepArgs& a, const SegTable& tb, const uint32_t* keys, const uint32_t* vals,
-                int64_t range, int64_t n_warps, SegRecords rec, DevStats* stats,
-                uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, cudaStream_t s) {
+template <int EPL, bool VECOK>
+int64_t launch_cfg(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
+                   const uint32_t* vals, SegRecords rec, int64_t max_warps, DevStats* stats,
+                   uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
+                   cudaStream_t s) {
+  constexpr size_t smem = seg_dyn_smem<EPL>();
+  static int blocks_per_sm = 0;  // static + dynamic shared memory may pass 48 KB
+  if (blocks_per_sm == 0) {
+    cudaFuncSetAttribute(k_segsum_apply<EPL, VECOK>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, k_segsum_apply<EPL, VECOK>, SEG_THREADS,
+                                                      smem) != cudaSuccess || b < 1)
+      b = 1;
+    blocks_per_sm = b;
+  }
+  // One wave of resident warps, each owning an equal range of whole rounds.
+  const int64_t Nt = tb.pos_end - tb.pos_begin;
+  int64_t target = (int64_t)num_sms * blocks_per_sm * SEG_WARPS;
+  if (target > max_warps) target = max_warps;
+  int64_t range = (Nt + target - 1) / target;
+  range = ((range + RS - 1) / RS) * RS;
+  if (range < RS) range = RS;
+  const int64_t n_warps = (Nt + range - 1) / range;
   const int64_t grid = (n_warps + SEG_WARPS - 1) / SEG_WARPS;
-  k_segsum_apply<VEC, L, EPL><<<(unsigned)grid, SEG_THREADS, 0, s>>>(
+  k_segsum_apply<EPL, VECOK><<<(unsigned)grid, SEG_THREADS, smem, s>>>(
       a, tb, keys, vals, range, n_warps, rec, stats, dbg_count, dbg_kept, err);
+  return n_warps;
+}
+
+
+template <int EPL>
+int64_t launch_rows(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
+                    const uint32_t* vals, SegRecords rec, int64_t max_warps, DevStats* stats,
+                    uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
+                    cudaStream_t s) {
+  constexpr size_t smem = rows_dyn_smem<EPL>();
+  static int blocks_per_sm = 0;
+  if (blocks_per_sm == 0) {
+    cudaFuncSetAttribute(k_segsum_rows<EPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, k_segsum_rows<EPL>, SEG_THREADS,
+                                                      smem) != cudaSuccess || b < 1)
+      b = 1;
+    blocks_per_sm = b;
+  }
+  const int64_t Nt = tb.pos_end - tb.pos_begin;
+  int64_t target = (int64_t)num_sms * blocks_per_sm * SEG_WARPS;
+  if (target > max_warps) target = max_warps;
+  int64_t range = (Nt + target - 1) / target;
+  range = ((range + RS - 1) / RS) * RS;
+  if (range < RS) range = RS;
+  const int64_t n_warps = (Nt + range - 1) / range;
+  const int64_t grid = (n_warps + SEG_WARPS - 1) / SEG_WARPS;
+  k_segsum_rows<EPL><<<(unsigned)grid, SEG_THREADS, smem, s>>>(a, tb, keys, vals, range, n_warps,
+                                                               rec, stats, dbg_count, dbg_kept,
+                                                               err);
+  return n_warps;
 }
 
 }  // namespace
 
-// Lane layout for a row width: 16-byte vectors when d is a multiple of 4,
-// L lanes per row (a power of two), EPL vectors per lane.
-void launch_segsum(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
-                   const uint32_t* vals, int64_t range, int64_t n_warps, SegRecords rec,
-                   DevStats* stats, uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err,
-                   int /*num_sms*/, cudaStream_t s) {
+// Rows of up to 64 floats take the lane-parallel kernel; wider rows the
+// warp-per-element one (EPL = elements per lane, vector accesses when d is a
+// multiple of EPL).  Returns the number of warp ranges (the fixup kernel's work).
+int64_t launch_segsum(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
+                      const uint32_t* vals, SegRecords rec, int64_t max_warps, DevStats* stats,
+                      uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
+                      cudaStream_t s) {
   const int d = tb.d;
-#define GBA_SEG(V, LL, EP) \
-  launch_cfg<V, LL, EP>(a, tb, keys, vals, range, n_warps, rec, stats, dbg_count, dbg_kept, err, s)
-  if (d % 4 == 0) {
-    const int units = d / 4;
-    if (units <= 1) GBA_SEG(4, 1, 1);
-    else if (units <= 2) GBA_SEG(4, 2, 1);
-    else if (units <= 4) GBA_SEG(4, 4, 1);
-    else if (units <= 8) GBA_SEG(4, 8, 1);
-    else if (units <= 16) GBA_SEG(4, 16, 1);
-    else if (units <= 32) GBA_SEG(4, 32, 1);
-    else GBA_SEG(4, 32, 2);
-  } else {
-    if (d <= 2) GBA_SEG(1, 2, 1);
-    else if (d <= 4) GBA_SEG(1, 4, 1);
-    else if (d <= 8) GBA_SEG(1, 8, 1);
-    else if (d <= 16) GBA_SEG(1, 16, 1);
-    else if (d <= 32) GBA_SEG(1, 32, 1);
-    else if (d <= 64) GBA_SEG(1, 32, 2);
-    else if (d <= 128) GBA_SEG(1, 32, 4);
-    else GBA_SEG(1, 32, 8);
+  if (d <= 32)
+    return launch_rows<1>(a, tb, keys, vals, rec, max_warps, stats, dbg_count, dbg_kept, err,
+                          num_sms, s);
+  if (d <= 64)
+    return launch_rows<2>(a, tb, keys, vals, rec, max_warps, stats, dbg_count, dbg_kept, err,
+                          num_sms, s);
+#define GBA_SEG(EP, VO)                                                                        \
+  return launch_cfg<EP, VO>(a, tb, keys, vals, rec, max_warps, stats, dbg_count, dbg_kept, err, \
+                            num_sms, s)
+  if (d <= 128) {
+    if (d % 4 == 0) GBA_SEG(4, true);
+    GBA_SEG(4, false);
   }
+  if (d % 8 == 0) GBA_SEG(8, true);
+  GBA_SEG(8, false);
 #undef GBA_SEG
 }
 

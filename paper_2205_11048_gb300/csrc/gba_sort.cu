@@ -25,6 +25,17 @@ constexpr int SORT_ITEMS = 16;
 constexpr int SORT_TILE = SORT_THREADS * SORT_ITEMS;
 constexpr int MAX_PASSES = 4;
 constexpr int LB_WIN = 8;  // look-back window
+constexpr int OFF_CACHE = 1024;  // message offsets kept in shared memory
+
+// Copies the step's message offsets into shared memory when they fit;
+// returns the array the key computation should read.
+__device__ __forceinline__ const uint32_t* cache_offsets(const StepArgs& a, uint32_t* s_off) {
+  const int n = a.T * (a.M + 1);
+  if (n > OFF_CACHE) return a.msg_off;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) s_off[i] = a.msg_off[i];
+  __syncthreads();
+  return s_off;
+}
 
 // Look-back status word: [63:32] epoch of the launch, [31:30] flag, [29:0] count.
 constexpr unsigned long long FLAG_AGG = 1ull << 30;
@@ -52,14 +63,22 @@ __device__ __forceinline__ uint32_t lanemask_lt() {
 // Key of global occurrence o: the table holding o, the message holding it, the
 // id, and the row it maps to (DIRECT ids outside [0, V) latch ERR_ID_RANGE and
 // are clamped to row 0; the whole step is then skipped by later kernels).
-__device__ __forceinline__ uint32_t occurrence_key(const StepArgs& a, int64_t o,
-                                                   const ErrSink& err) {
+__device__ __forceinline__ uint32_t occurrence_key(const StepArgs& a, const uint32_t* offs,
+                                                   int64_t o, const ErrSink& err) {
   int t = 0;
   while (t + 1 < a.T && __ldg(a.nbase + t + 1) <= o) ++t;
   const uint32_t ot = (uint32_t)(o - __ldg(a.nbase + t));
-  const uint32_t* off = a.msg_off + (size_t)t * (a.M + 1);
-  const int m = message_of(off, a.M, ot);
-  const uint32_t p = ot - __ldg(off + m);
+  const uint32_t* off = offs + (size_t)t * (a.M + 1);
+  int lo = 0, hi = a.M;  // the message holding ot: off[lo] <= ot < off[lo + 1]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (off[mid] <= ot)
+      lo = mid;
+    else
+      hi = mid;
+  }
+  const int m = lo;
+  const uint32_t p = ot - off[m];
   const int64_t* ids = a.ids_ptr[(size_t)t * a.M + m];
   const int64_t id = __ldg(ids + p);
   const TableInfo ti = a.tinfo[t];
@@ -148,11 +167,13 @@ __global__ void __launch_bounds__(256) k_message_weights(StepArgs a, StepScratch
 __global__ void __launch_bounds__(SORT_THREADS) k_sort_histogram(StepArgs a, int passes,
                                                                  StepScratch sc, ErrSink err) {
   __shared__ uint32_t h[MAX_PASSES][RADIX];
+  __shared__ uint32_t s_off[OFF_CACHE];
   for (int i = threadIdx.x; i < MAX_PASSES * RADIX; i += SORT_THREADS) (&h[0][0])[i] = 0u;
+  const uint32_t* offs = cache_offsets(a, s_off);
   __syncthreads();
   const int64_t stride = (int64_t)gridDim.x * SORT_THREADS;
   for (int64_t o = (int64_t)blockIdx.x * SORT_THREADS + threadIdx.x; o < a.N; o += stride) {
-    const uint32_t key = occurrence_key(a, o, err);
+    const uint32_t key = occurrence_key(a, offs, o, err);
     for (int p = 0; p < passes; ++p) atomicAdd(&h[p][(key >> (8 * p)) & (RADIX - 1)], 1u);
   }
   __syncthreads();
@@ -178,6 +199,7 @@ __global__ void __launch_bounds__(SORT_THREADS)
   __shared__ uint32_t s_keys[SORT_TILE];
   __shared__ uint32_t s_vals[SORT_TILE];
   __shared__ uint32_t s_tile;
+  __shared__ uint32_t s_off[FIRST ? OFF_CACHE : 1];
 
   // An id range error was latched before this launch (by the histogram):
   // every tile of every pass skips, consistently.
@@ -188,6 +210,7 @@ __global__ void __launch_bounds__(SORT_THREADS)
   for (int i = tid; i < SORT_WARPS * RADIX; i += SORT_THREADS) (&s_warp[0][0])[i] = 0u;
   __syncthreads();
 
+  const uint32_t* offs = FIRST ? cache_offsets(a, s_off) : nullptr;
   const uint32_t tile = s_tile;
   const int64_t N = a.N;
   const int64_t base = (int64_t)tile * SORT_TILE;
@@ -199,7 +222,7 @@ __global__ void __launch_bounds__(SORT_THREADS)
     const int64_t idx = base + (int64_t)warp * (SORT_ITEMS * 32) + j * 32 + lane;
     if (idx < N) {
       if (FIRST) {
-        key[j] = occurrence_key(a, idx, err);
+        key[j] = occurrence_key(a, offs, idx, err);
         val[j] = (uint32_t)idx;
       } else {
         key[j] = keys_in[idx];

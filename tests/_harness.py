@@ -179,3 +179,61 @@ def run_parity(cfg: W.WorkloadCfg, steps: int, tol: float, by_ref=False, check_e
     assert g.version() == steps == orc.pull_version()
     g.close()
     return worst
+
+
+def rows_of_gpu(tb, ids: torch.Tensor) -> torch.Tensor:
+    """Row of each id (int64 tensor on the device): DIRECT ids as they are,
+    MODULO ids by the residue of their unsigned 64-bit value."""
+    if tb.id_mode == W.DIRECT:
+        return ids
+    V = tb.rows
+    r = torch.remainder(ids, V)
+    wrap = (1 << 64) % V            # 2^64 mod V, added for negative ids
+    return torch.where(ids < 0, torch.remainder(r + wrap, V), r)
+
+
+def run_fullsize(cfg: W.WorkloadCfg, steps: int, tol: float, n_hot=150, n_rand=1500,
+                 n_dense=20000, seed=0):
+    """Full-size workload in the benchmark's launch configuration (messages
+    pushed by reference), checked against the oracle on a sample of rows (hot
+    and random rows touched by the first step) and of dense parameters."""
+    g = make_gpu(cfg, debug=False)
+    gen = torch.Generator().manual_seed(seed)
+    first = W.generate_step(cfg, 0, "cuda")
+    track = []
+    for t, tb in enumerate(cfg.tables):
+        rows = torch.cat([rows_of_gpu(tb, m["ids"][t]) for m in first])
+        u, cnt = torch.unique(rows, return_counts=True)
+        hot = u[torch.argsort(cnt, descending=True)[:n_hot]]
+        pick = torch.randperm(u.numel(), generator=gen)[:n_rand].to(u.device)
+        rnd = u[pick]
+        cold = torch.randint(0, tb.rows, (50,), generator=gen).to(u.device)
+        track.append(torch.unique(torch.cat([hot, rnd, cold])))
+    dense_idx = torch.unique(torch.cat([
+        torch.randint(0, cfg.D, (n_dense,), generator=gen),
+        torch.tensor([0, 1, 2, 3, cfg.D - 1, cfg.D - 2]).clamp(0, cfg.D - 1)]))
+    orc = make_oracle(cfg, track_rows=[t.cpu().numpy() for t in track],
+                      track_dense=dense_idx.numpy())
+    dense_host = [np.zeros(cfg.D, np.float32) for _ in range(cfg.M)]
+    dense_dev_idx = dense_idx.to("cuda")
+    for k in range(steps):
+        msgs = first if k == 0 else W.generate_step(cfg, k, "cuda")
+        for i, m in enumerate(msgs):
+            push_gpu(g, m, by_ref=True)
+            ids_f, rows_f = [], []
+            for t, tb in enumerate(cfg.tables):
+                sel = torch.isin(rows_of_gpu(tb, m["ids"][t]), track[t])
+                ids_f.append(m["ids"][t][sel].cpu().numpy())
+                rows_f.append(m["rows"][t][sel].cpu().numpy())
+            dh = dense_host[i]
+            dh[dense_idx.numpy()] = m["dense"][dense_dev_idx].cpu().numpy()
+            orc.push(O.Message(int(m["token"]), int(m["local_batch"]), ids_f, rows_f, dh.copy()))
+        assert g.try_apply() == 1
+        assert orc.try_apply() == 1
+        g.sync()
+        keep_g = g.keep()
+        assert np.array_equal(keep_g, orc.last_keep), "message weights differ"
+        msgs = None
+    worst = compare_state(g, orc, tol)
+    g.close()
+    return worst
