@@ -199,6 +199,17 @@ const char* gba_last_error(gba_handle* h);
 /* gba_destroy - wait for outstanding work and free everything (NULL is a no-op). */
 void gba_destroy(gba_handle* h);
 
+/*
+ * gba_set_overlap - when on, gba_try_apply does not order the handle's stream
+ * after the step it enqueues, so the next step's message weights and sort can
+ * run while this step's segment-sum and dense update finish (steps still apply
+ * in order: each step's row update follows the previous one's).  The caller
+ * then sees a step's results after gba_sync (or any call that synchronises).
+ * Copying pushes still wait for every earlier step.  Default off: every step is
+ * complete, in the handle's stream order, before later work on that stream.
+ */
+gba_status gba_set_overlap(gba_handle* h, int32_t on);
+
 /* ---- instrumentation and test entry points ----------------------------- */
 
 /* gba_set_timing - when on, every kernel launch is bracketed by CUDA events on

@@ -96,6 +96,7 @@ _SIGNATURES = {
     "gba_set_timing": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_kernel_times": (ctypes.c_int, [_P, ctypes.POINTER(gba_kernel_times_t)]),
     "gba_set_debug": (ctypes.c_int, [_P, ctypes.c_int32]),
+    "gba_set_overlap": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_debug_segments": (ctypes.c_int, [_P, ctypes.c_int64, _P, _P, _P, _P,
                                           ctypes.POINTER(ctypes.c_int64)]),
     "gba_debug_sorted": (ctypes.c_int, [_P, ctypes.c_int64, _P, _P,
@@ -306,6 +307,9 @@ class GBA:
         s = gba_stats_t()
         check(self.L.gba_stats(self.h, ctypes.byref(s)), self.h)
         return s.as_dict()
+
+    def set_overlap(self, on=True):
+        check(self.L.gba_set_overlap(self.h, int(on)), self.h)
 
     def set_debug(self, on=True):
         check(self.L.gba_set_debug(self.h, int(on)), self.h)

@@ -82,7 +82,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
   uint64_t* empty = full + STAGES;
   __shared__ int s_abort;
 
-  if (*(volatile uint32_t*)err.dev & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  if (*(volatile uint32_t*)err.step & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) {

@@ -23,6 +23,9 @@ constexpr int MAX_DIM = 256;
 constexpr int META_SLOTS = 4;
 constexpr int MAX_PASSES = 4;
 constexpr int64_t MAX_STEP_OCC = (1ll << 30) - 1;
+// Per-step buffers exist twice, so that step k + 1's message weights and sort
+// run (on the sort stream) while step k's segment-sum and dense update run.
+constexpr int SLOTS = 2;
 
 struct Arena {  // contiguous-allocation ring over [0, cap) with virtual offsets
   int64_t cap = 0;
@@ -77,8 +80,14 @@ struct gba_handle {
   int num_sms = 152;
   cudaStream_t stream = nullptr;
   bool own_stream = false;
-  cudaStream_t side = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  cudaStream_t side = nullptr;   // dense update
+  cudaStream_t sorts = nullptr;   // message weights, histogram, sort passes
+  cudaStream_t applys = nullptr;  // segment-sum and row update
+  bool overlap = false;           // consecutive steps may run concurrently
+  cudaEvent_t ev_pushes = nullptr;
+  cudaEvent_t ev_hist[SLOTS] = {}, ev_sorted[SLOTS] = {}, ev_applied[SLOTS] = {},
+              ev_densed[SLOTS] = {};
+  bool slot_busy[SLOTS] = {};
 
   std::vector<TableState> tables;
   int32_t T = 0;
@@ -106,23 +115,23 @@ struct gba_handle {
   std::vector<TableInfo> h_tinfo;
 
   size_t meta_bytes = 0;
-  char* d_meta = nullptr;
+  char* d_meta[SLOTS] = {};
   char* h_meta[META_SLOTS] = {};
   cudaEvent_t meta_ev[META_SLOTS] = {};
   int meta_slot = 0;
 
   // sort / segment scratch, grown on demand
   int64_t n_cap = 0;
-  uint32_t* d_keys[2] = {};
-  uint32_t* d_vals[2] = {};
-  unsigned long long* d_status = nullptr;
+  uint32_t* d_keys[SLOTS][2] = {};
+  uint32_t* d_vals[SLOTS][2] = {};
+  unsigned long long* d_status[SLOTS] = {};
   int64_t status_tiles = 0;
   uint32_t epoch = 0;
   uint32_t* d_dbg_count = nullptr;
   uint32_t* d_dbg_kept = nullptr;
   int64_t dbg_cap = 0;
-  char* d_step_scratch = nullptr;
-  StepScratch sc{};
+  char* d_step_scratch[SLOTS] = {};
+  StepScratch sc[SLOTS] = {};
   SegRecords rec{};
   int64_t rec_warps = 0;
   int d_max = 1;
@@ -146,6 +155,7 @@ struct gba_handle {
   bool have_last = false;
   int64_t last_N = 0;
   int last_buf = 0;
+  int last_slot = 0;
   int32_t last_M = 0;
 };
 
@@ -240,8 +250,10 @@ OptStep make_opt_step(const gba_opt_desc& o, double bpow1_next, double bpow2_nex
 void free_all(gba_handle* h) {
   if (!h) return;
   cudaSetDevice(h->device);
-  if (h->stream) cudaStreamSynchronize(h->stream);
+  if (h->sorts) cudaStreamSynchronize(h->sorts);
+  if (h->applys) cudaStreamSynchronize(h->applys);
   if (h->side) cudaStreamSynchronize(h->side);
+  if (h->stream) cudaStreamSynchronize(h->stream);
   for (auto& t : h->tables) {
     cudaFree(t.w);
     cudaFree(t.s0);
@@ -255,19 +267,23 @@ void free_all(gba_handle* h) {
   cudaFree(h->ds1);
   cudaFree(h->dense_ring);
   cudaFree(h->d_tinfo);
-  cudaFree(h->d_meta);
+  for (int b = 0; b < SLOTS; ++b) {
+    cudaFree(h->d_meta[b]);
+    cudaFree(h->d_step_scratch[b]);
+    cudaFree(h->d_status[b]);
+    for (int i = 0; i < 2; ++i) {
+      cudaFree(h->d_keys[b][i]);
+      cudaFree(h->d_vals[b][i]);
+    }
+    for (cudaEvent_t e : {h->ev_hist[b], h->ev_sorted[b], h->ev_applied[b], h->ev_densed[b]})
+      if (e) cudaEventDestroy(e);
+  }
   for (int i = 0; i < META_SLOTS; ++i) {
     if (h->h_meta[i]) cudaFreeHost(h->h_meta[i]);
     if (h->meta_ev[i]) cudaEventDestroy(h->meta_ev[i]);
   }
-  for (int i = 0; i < 2; ++i) {
-    cudaFree(h->d_keys[i]);
-    cudaFree(h->d_vals[i]);
-  }
-  cudaFree(h->d_status);
   cudaFree(h->d_dbg_count);
   cudaFree(h->d_dbg_kept);
-  cudaFree(h->d_step_scratch);
   cudaFree(h->rec.hi);
   cudaFree(h->rec.lo);
   cudaFree(h->rec.meta);
@@ -279,18 +295,35 @@ void free_all(gba_handle* h) {
     cudaEventDestroy(p.b);
   }
   for (auto e : h->event_pool) cudaEventDestroy(e);
-  if (h->ev_fork) cudaEventDestroy(h->ev_fork);
-  if (h->ev_join) cudaEventDestroy(h->ev_join);
+  if (h->ev_pushes) cudaEventDestroy(h->ev_pushes);
   if (h->side) cudaStreamDestroy(h->side);
+  if (h->sorts) cudaStreamDestroy(h->sorts);
+  if (h->applys) cudaStreamDestroy(h->applys);
   if (h->own_stream && h->stream) cudaStreamDestroy(h->stream);
+}
+
+cudaError_t sync_all(gba_handle* h) {
+  cudaError_t e[4] = {cudaStreamSynchronize(h->sorts), cudaStreamSynchronize(h->applys),
+                      cudaStreamSynchronize(h->side), cudaStreamSynchronize(h->stream)};
+  for (cudaError_t x : e)
+    if (x != cudaSuccess) return x;
+  return cudaSuccess;
+}
+
+// Orders the handle's stream after every step enqueued so far.
+void join_steps(gba_handle* h) {
+  for (int b = 0; b < SLOTS; ++b)
+    if (h->slot_busy[b]) {
+      cudaStreamWaitEvent(h->stream, h->ev_applied[b], 0);
+      cudaStreamWaitEvent(h->stream, h->ev_densed[b], 0);
+    }
 }
 
 // Device error latched by a kernel?  Polls the mapped flag without
 // synchronising; if set, synchronises and turns the word into a status.
 gba_status poll_device_error(gba_handle* h, bool force_sync) {
   if (!force_sync && *(volatile uint32_t*)h->h_err == 0u) return GBA_OK;
-  cudaStreamSynchronize(h->side);
-  cudaError_t e = cudaStreamSynchronize(h->stream);
+  cudaError_t e = sync_all(h);
   if (e != cudaSuccess) {
     h->failed = true;
     h->fail_code = cuda_fail(h, e, "stream synchronize");
@@ -317,26 +350,28 @@ gba_status poll_device_error(gba_handle* h, bool force_sync) {
 
 gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
   if (N > h->n_cap) {
-    cudaStreamSynchronize(h->side);
-    cudaStreamSynchronize(h->stream);
+    sync_all(h);
     int64_t cap = std::max<int64_t>(N + N / 4, 4096);
-    for (int i = 0; i < 2; ++i) {
-      cudaFree(h->d_keys[i]);
-      cudaFree(h->d_vals[i]);
-      h->d_keys[i] = h->d_vals[i] = nullptr;
-      GBA_CUDA(h, cudaMalloc(&h->d_keys[i], cap * sizeof(uint32_t)));
-      GBA_CUDA(h, cudaMalloc(&h->d_vals[i], cap * sizeof(uint32_t)));
+    const int64_t tiles = sort_tiles(cap);
+    for (int b = 0; b < SLOTS; ++b) {
+      for (int i = 0; i < 2; ++i) {
+        cudaFree(h->d_keys[b][i]);
+        cudaFree(h->d_vals[b][i]);
+        h->d_keys[b][i] = h->d_vals[b][i] = nullptr;
+        GBA_CUDA(h, cudaMalloc(&h->d_keys[b][i], cap * sizeof(uint32_t)));
+        GBA_CUDA(h, cudaMalloc(&h->d_vals[b][i], cap * sizeof(uint32_t)));
+      }
+      cudaFree(h->d_status[b]);
+      h->d_status[b] = nullptr;
+      GBA_CUDA(h, cudaMalloc(&h->d_status[b], (size_t)tiles * 256 * sizeof(unsigned long long)));
+      GBA_CUDA(h,
+               cudaMemset(h->d_status[b], 0, (size_t)tiles * 256 * sizeof(unsigned long long)));
     }
     h->n_cap = cap;
-    const int64_t tiles = sort_tiles(cap);
-    cudaFree(h->d_status);
-    h->d_status = nullptr;
-    GBA_CUDA(h, cudaMalloc(&h->d_status, (size_t)tiles * 256 * sizeof(unsigned long long)));
-    GBA_CUDA(h, cudaMemset(h->d_status, 0, (size_t)tiles * 256 * sizeof(unsigned long long)));
     h->status_tiles = tiles;
   }
   if (h->debug && N > h->dbg_cap) {
-    cudaStreamSynchronize(h->stream);
+    sync_all(h);
     cudaFree(h->d_dbg_count);
     cudaFree(h->d_dbg_kept);
     h->d_dbg_count = h->d_dbg_kept = nullptr;
@@ -401,6 +436,8 @@ gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_
   if (copy) {
     gba_status s = ensure_arenas(h);
     if (s != GBA_OK) return s;
+    // The copy may overwrite buffer space of messages that earlier steps read.
+    if (h->overlap) join_steps(h);
     if (h->D > 0 && h->slot_count >= h->max_buf)
       return set_err(h, GBA_E_FULL, "gradient buffer full");
     std::vector<int64_t> saved_tail(h->T);
@@ -514,9 +551,14 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
     h->own_stream = true;
   }
   if (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming) != cudaSuccess)
+      cudaStreamCreateWithFlags(&h->sorts, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaStreamCreateWithFlags(&h->applys, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_pushes, cudaEventDisableTiming) != cudaSuccess)
     return fail(GBA_E_CUDA);
+  for (int b = 0; b < SLOTS; ++b)
+    for (cudaEvent_t* e : {&h->ev_hist[b], &h->ev_sorted[b], &h->ev_applied[b], &h->ev_densed[b]})
+      if (cudaEventCreateWithFlags(e, cudaEventDisableTiming) != cudaSuccess)
+        return fail(GBA_E_CUDA);
   if (configure_dense() != cudaSuccess) return fail(GBA_E_CUDA);
 
   // key space: tables in order
@@ -567,7 +609,8 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
     const size_t M = (size_t)max_buffered_msgs, T = (size_t)n_tables;
     h->meta_bytes = align16(M * 8) + align16(M * 8) + align16(T * (M + 1) * 4) +
                     align16(T * M * 8) + align16(T * M * 8) + align16((T + 1) * 8);
-    if (!dev_alloc((void**)&h->d_meta, h->meta_bytes)) return fail(GBA_E_OOM);
+    for (int b = 0; b < SLOTS; ++b)
+      if (!dev_alloc((void**)&h->d_meta[b], h->meta_bytes)) return fail(GBA_E_OOM);
     for (int i = 0; i < META_SLOTS; ++i) {
       if (cudaHostAlloc((void**)&h->h_meta[i], h->meta_bytes, cudaHostAllocDefault) !=
               cudaSuccess ||
@@ -578,18 +621,24 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   {
     const size_t M = (size_t)max_buffered_msgs;
     const size_t bytes = align16(MAX_PASSES * 256 * 4) + align16(MAX_PASSES * 4) +
-                         align16(M * 4) + align16(M * 4) + align16(4);
-    if (!dev_alloc((void**)&h->d_step_scratch, bytes)) return fail(GBA_E_OOM);
-    char* p = h->d_step_scratch;
-    h->sc.hist = (uint32_t*)p;
-    p += align16(MAX_PASSES * 256 * 4);
-    h->sc.tile_counter = (uint32_t*)p;
-    p += align16(MAX_PASSES * 4);
-    h->sc.keep = (int32_t*)p;
-    p += align16(M * 4);
-    h->sc.kept_list = (int32_t*)p;
-    p += align16(M * 4);
-    h->sc.n_kept = (int32_t*)p;
+                         align16(M * 4) + align16(M * 4) + align16(4) + align16(4);
+    for (int b = 0; b < SLOTS; ++b) {
+      if (!dev_alloc((void**)&h->d_step_scratch[b], bytes)) return fail(GBA_E_OOM);
+      if (cudaMemset(h->d_step_scratch[b], 0, bytes) != cudaSuccess) return fail(GBA_E_CUDA);
+      char* p = h->d_step_scratch[b];
+      StepScratch& sc = h->sc[b];
+      sc.hist = (uint32_t*)p;
+      p += align16(MAX_PASSES * 256 * 4);
+      sc.tile_counter = (uint32_t*)p;
+      p += align16(MAX_PASSES * 4);
+      sc.keep = (int32_t*)p;
+      p += align16(M * 4);
+      sc.kept_list = (int32_t*)p;
+      p += align16(M * 4);
+      sc.n_kept = (int32_t*)p;
+      p += align16(4);
+      sc.step_err = (uint32_t*)p;
+    }
   }
   {
     h->rec_warps = (int64_t)h->num_sms * 64 + 64;
@@ -606,7 +655,7 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   uint32_t* h_err_dev = nullptr;
   if (cudaHostGetDevicePointer((void**)&h_err_dev, h->h_err, 0) != cudaSuccess)
     return fail(GBA_E_CUDA);
-  h->sink = ErrSink{h->d_err, h_err_dev};
+  h->sink = ErrSink{nullptr, h->d_err, h_err_dev};  // .step is set per slot
   if (cudaMemsetAsync(h->d_err, 0, 4, h->stream) != cudaSuccess ||
       cudaMemsetAsync(h->d_stats, 0, sizeof(DevStats), h->stream) != cudaSuccess)
     return fail(GBA_E_CUDA);
@@ -674,6 +723,22 @@ int32_t gba_try_apply(gba_handle* h) {
     if (s != GBA_OK) return s;
   }
 
+  // ---- the step's buffers (slot b) and stream dependencies.  The sort stream
+  // runs message weights, histogram and sort passes; the handle's stream the
+  // segment-sum and row update; the side stream the dense update.
+  const int b = (int)(h->k & 1);
+  // everything the caller enqueued before this call (pushes included)
+  cudaEventRecord(h->ev_pushes, h->stream);
+  cudaStreamWaitEvent(h->sorts, h->ev_pushes, 0);
+  if (h->slot_busy[b]) {  // step k - 2 used these buffers
+    cudaStreamWaitEvent(h->sorts, h->ev_applied[b], 0);
+    cudaStreamWaitEvent(h->sorts, h->ev_densed[b], 0);
+  }
+  StepScratch& sc = h->sc[b];
+  ErrSink sink = h->sink;
+  sink.step = sc.step_err;
+  char* dmeta = h->d_meta[b];
+
   // ---- step descriptor
   const int slot = h->meta_slot;
   h->meta_slot = (h->meta_slot + 1) % META_SLOTS;
@@ -712,8 +777,8 @@ int32_t gba_try_apply(gba_handle* h) {
     moff[(size_t)t * (M + 1) + M] = run;
   }
   for (int t = 0; t <= T; ++t) nb[t] = nbase[t];
-  GBA_CUDA(h, cudaMemcpyAsync(h->d_meta, hp, h->meta_bytes, cudaMemcpyHostToDevice, h->stream));
-  cudaEventRecord(h->meta_ev[slot], h->stream);
+  GBA_CUDA(h, cudaMemcpyAsync(dmeta, hp, h->meta_bytes, cudaMemcpyHostToDevice, h->sorts));
+  cudaEventRecord(h->meta_ev[slot], h->sorts);
 
   StepArgs a{};
   a.k = h->k;
@@ -723,18 +788,18 @@ int32_t gba_try_apply(gba_handle* h) {
   a.iota = h->st.iota;
   a.row_staleness = h->st.row_staleness;
   a.sparse_den = h->st.sparse_denominator;
-  a.tokens = (const int64_t*)(h->d_meta + o_tok);
-  a.dense_ptr = (const float* const*)(h->d_meta + o_dense);
-  a.msg_off = (const uint32_t*)(h->d_meta + o_off);
-  a.ids_ptr = (const int64_t* const*)(h->d_meta + o_ids);
-  a.rows_ptr = (const float* const*)(h->d_meta + o_rows);
-  a.nbase = (const int64_t*)(h->d_meta + o_nbase);
+  a.tokens = (const int64_t*)(dmeta + o_tok);
+  a.dense_ptr = (const float* const*)(dmeta + o_dense);
+  a.msg_off = (const uint32_t*)(dmeta + o_off);
+  a.ids_ptr = (const int64_t* const*)(dmeta + o_ids);
+  a.rows_ptr = (const float* const*)(dmeta + o_rows);
+  a.nbase = (const int64_t*)(dmeta + o_nbase);
   a.tinfo = h->d_tinfo;
 
   // ---- K1: message weights (Eq. (1)); clears the per-step scratch
   {
-    Timed tm(h, GBA_K_WEIGHTS, h->stream);
-    launch_weights(a, h->sc, h->d_stats, MAX_PASSES * 256, h->stream);
+    Timed tm(h, GBA_K_WEIGHTS, h->sorts);
+    launch_weights(a, sc, h->d_stats, MAX_PASSES * 256, h->sorts);
   }
   // ---- K5 on the side stream, concurrently with the sort and segment-sum.
   // It is forked after the histogram kernel has validated every id, so a step
@@ -744,13 +809,12 @@ int32_t gba_try_apply(gba_handle* h) {
     const double p1 = h->dbpow1 * (double)h->dense_opt.beta1;
     const double p2 = h->dbpow2 * (double)h->dense_opt.beta2;
     DenseArgs da{h->dw, h->ds0, h->ds1, h->D, M, make_opt_step(h->dense_opt, p1, p2)};
-    cudaEventRecord(h->ev_fork, h->stream);
-    cudaStreamWaitEvent(h->side, h->ev_fork, 0);
+    cudaEventRecord(h->ev_hist[b], h->sorts);
+    cudaStreamWaitEvent(h->side, h->ev_hist[b], 0);
     {
       Timed tm(h, GBA_K_DENSE, h->side);
-      launch_dense(a, da, h->sc, h->sink, h->wait_ns, h->num_sms, h->side);
+      launch_dense(a, da, sc, sink, h->wait_ns, h->num_sms, h->side);
     }
-    cudaEventRecord(h->ev_join, h->side);
     h->dbpow1 = p1;
     h->dbpow2 = p2;
   };
@@ -758,9 +822,9 @@ int32_t gba_try_apply(gba_handle* h) {
   int final_buf = 0;
   if (N > 0) {
     {
-      Timed tm(h, GBA_K_SORT_HIST, h->stream);
+      Timed tm(h, GBA_K_SORT_HIST, h->sorts);
       int grid = (int)std::min<int64_t>((N + 255) / 256, (int64_t)h->num_sms * 8);
-      launch_sort_histogram(a, h->passes, h->sc, h->sink, std::max(grid, 1), h->stream);
+      launch_sort_histogram(a, h->passes, sc, sink, std::max(grid, 1), h->sorts);
     }
     launch_dense_side();
     const uint32_t* kin = nullptr;
@@ -768,13 +832,15 @@ int32_t gba_try_apply(gba_handle* h) {
     for (int p = 0; p < h->passes; ++p) {
       const int ob = p & 1;
       if (++h->epoch == 0u) h->epoch = 1u;
-      Timed tm(h, GBA_K_SORT_PASS, h->stream);
-      launch_onesweep(a, p == 0, p, kin, vin, h->d_keys[ob], h->d_vals[ob], h->sc, h->d_status,
-                      h->epoch, h->sink, h->wait_ns, h->stream);
-      kin = h->d_keys[ob];
-      vin = h->d_vals[ob];
+      Timed tm(h, GBA_K_SORT_PASS, h->sorts);
+      launch_onesweep(a, p == 0, p, kin, vin, h->d_keys[b][ob], h->d_vals[b][ob], sc,
+                      h->d_status[b], h->epoch, sink, h->wait_ns, h->sorts);
+      kin = h->d_keys[b][ob];
+      vin = h->d_vals[b][ob];
       final_buf = ob;
     }
+    cudaEventRecord(h->ev_sorted[b], h->sorts);
+    cudaStreamWaitEvent(h->applys, h->ev_sorted[b], 0);
     for (int t = 0; t < T; ++t) {
       const int64_t Nt = nbase[t + 1] - nbase[t];
       if (Nt == 0) continue;
@@ -797,23 +863,33 @@ int32_t gba_try_apply(gba_handle* h) {
       uint32_t* dk = h->debug ? h->d_dbg_kept : nullptr;
       int64_t n_warps = 0;
       {
-        Timed tm(h, GBA_K_SEGSUM, h->stream);
-        n_warps = launch_segsum(a, tb, h->d_keys[final_buf], h->d_vals[final_buf], h->rec,
-                                h->rec_warps, h->d_stats, dc, dk, h->sink, h->num_sms, h->stream);
+        Timed tm(h, GBA_K_SEGSUM, h->applys);
+        n_warps = launch_segsum(a, tb, h->d_keys[b][final_buf], h->d_vals[b][final_buf],
+                                h->rec, h->rec_warps, h->d_stats, dc, dk, sink, h->num_sms,
+                                h->applys);
       }
       {
-        Timed tm(h, GBA_K_FIXUP, h->stream);
-        launch_fixup(a, tb, n_warps, h->rec, h->d_stats, dc, dk, h->sink, h->stream);
+        Timed tm(h, GBA_K_FIXUP, h->applys);
+        launch_fixup(a, tb, n_warps, h->rec, h->d_stats, dc, dk, sink, h->applys);
       }
     }
   }
-  if (N == 0) launch_dense_side();
+  if (N == 0) {
+    launch_dense_side();
+    cudaEventRecord(h->ev_sorted[b], h->sorts);
+    cudaStreamWaitEvent(h->applys, h->ev_sorted[b], 0);
+  }
   // Adam step counts advance every global step, whether or not a row moved.
   for (auto& ts : h->tables) {
     ts.bpow1 *= (double)ts.desc.opt.beta1;
     ts.bpow2 *= (double)ts.desc.opt.beta2;
   }
-  if (h->D > 0) cudaStreamWaitEvent(h->stream, h->ev_join, 0);
+  cudaEventRecord(h->ev_applied[b], h->applys);
+  cudaEventRecord(h->ev_densed[b], h->side);
+  h->slot_busy[b] = true;
+  // Unless steps may overlap, work the caller orders after this call on its
+  // stream sees the whole step.
+  if (!h->overlap) join_steps(h);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     h->failed = true;
@@ -838,6 +914,7 @@ int32_t gba_try_apply(gba_handle* h) {
   h->have_last = true;
   h->last_N = N;
   h->last_buf = final_buf;
+  h->last_slot = b;
   h->last_M = M;
   return 1;
 }
@@ -873,7 +950,7 @@ gba_status gba_get_dense(gba_handle* h, float** w, float** slot0, float** slot1)
 gba_status gba_stats(gba_handle* h, gba_stats_t* out) {
   if (!h || !out) return GBA_E_ARG;
   cudaSetDevice(h->device);
-  cudaStreamSynchronize(h->side);
+  sync_all(h);
   DevStats s{};
   GBA_CUDA(h, cudaMemcpyAsync(&s, h->d_stats, sizeof s, cudaMemcpyDeviceToHost, h->stream));
   GBA_CUDA(h, cudaStreamSynchronize(h->stream));
@@ -903,8 +980,7 @@ void gba_destroy(gba_handle* h) {
 
 gba_status gba_set_timing(gba_handle* h, int32_t on) {
   if (!h) return GBA_E_ARG;
-  cudaStreamSynchronize(h->side);
-  cudaStreamSynchronize(h->stream);
+  sync_all(h);
   collect_timing(h);
   h->times = gba_kernel_times_t{};
   h->timing = on != 0;
@@ -914,10 +990,17 @@ gba_status gba_set_timing(gba_handle* h, int32_t on) {
 gba_status gba_kernel_times(gba_handle* h, gba_kernel_times_t* out) {
   if (!h || !out) return GBA_E_ARG;
   cudaSetDevice(h->device);
-  cudaStreamSynchronize(h->side);
-  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  GBA_CUDA(h, sync_all(h));
   collect_timing(h);
   *out = h->times;
+  return GBA_OK;
+}
+
+gba_status gba_set_overlap(gba_handle* h, int32_t on) {
+  if (!h) return GBA_E_ARG;
+  cudaSetDevice(h->device);
+  if (!on) join_steps(h);
+  h->overlap = on != 0;
   return GBA_OK;
 }
 
@@ -933,12 +1016,11 @@ gba_status gba_debug_segments(gba_handle* h, int64_t cap, int32_t* table, int64_
   if (!h->have_last || !h->debug || !h->d_dbg_count)
     return set_err(h, GBA_E_STATE, "no debug record of a step (enable debug before the step)");
   cudaSetDevice(h->device);
-  cudaStreamSynchronize(h->side);
-  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  GBA_CUDA(h, sync_all(h));
   const int64_t N = h->last_N;
   std::vector<uint32_t> keys(N), cnt(N), kp(N);
   if (N > 0) {
-    GBA_CUDA(h, cudaMemcpy(keys.data(), h->d_keys[h->last_buf], N * 4, cudaMemcpyDeviceToHost));
+    GBA_CUDA(h, cudaMemcpy(keys.data(), h->d_keys[h->last_slot][h->last_buf], N * 4, cudaMemcpyDeviceToHost));
     GBA_CUDA(h, cudaMemcpy(cnt.data(), h->d_dbg_count, N * 4, cudaMemcpyDeviceToHost));
     GBA_CUDA(h, cudaMemcpy(kp.data(), h->d_dbg_kept, N * 4, cudaMemcpyDeviceToHost));
   }
@@ -964,15 +1046,14 @@ gba_status gba_debug_sorted(gba_handle* h, int64_t cap, uint32_t* keys, uint32_t
   if (!h || !n) return GBA_E_ARG;
   if (!h->have_last) return set_err(h, GBA_E_STATE, "no step applied yet");
   cudaSetDevice(h->device);
-  cudaStreamSynchronize(h->side);
-  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  GBA_CUDA(h, sync_all(h));
   *n = h->last_N;
   if (h->last_N > cap) return set_err(h, GBA_E_ARG, "capacity too small");
   if (h->last_N > 0) {
     if (keys)
-      GBA_CUDA(h, cudaMemcpy(keys, h->d_keys[h->last_buf], h->last_N * 4, cudaMemcpyDeviceToHost));
+      GBA_CUDA(h, cudaMemcpy(keys, h->d_keys[h->last_slot][h->last_buf], h->last_N * 4, cudaMemcpyDeviceToHost));
     if (occ)
-      GBA_CUDA(h, cudaMemcpy(occ, h->d_vals[h->last_buf], h->last_N * 4, cudaMemcpyDeviceToHost));
+      GBA_CUDA(h, cudaMemcpy(occ, h->d_vals[h->last_slot][h->last_buf], h->last_N * 4, cudaMemcpyDeviceToHost));
   }
   return GBA_OK;
 }
@@ -981,12 +1062,11 @@ gba_status gba_debug_keep(gba_handle* h, int32_t cap, int32_t* keep, int32_t* M)
   if (!h || !M) return GBA_E_ARG;
   if (!h->have_last) return set_err(h, GBA_E_STATE, "no step applied yet");
   cudaSetDevice(h->device);
-  cudaStreamSynchronize(h->side);
-  GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+  GBA_CUDA(h, sync_all(h));
   *M = h->last_M;
   if (h->last_M > cap) return set_err(h, GBA_E_ARG, "capacity too small");
   if (keep && h->last_M > 0)
-    GBA_CUDA(h, cudaMemcpy(keep, h->sc.keep, h->last_M * 4, cudaMemcpyDeviceToHost));
+    GBA_CUDA(h, cudaMemcpy(keep, h->sc[h->last_slot].keep, h->last_M * 4, cudaMemcpyDeviceToHost));
   return GBA_OK;
 }
 

@@ -11,14 +11,18 @@ constexpr uint32_t ERR_ID_RANGE = 1u;
 constexpr uint32_t ERR_TIMEOUT = 2u;
 constexpr uint32_t ERR_INTERNAL = 4u;
 
-// Where kernels report a failure: an atomic word in device memory plus a flag
-// in mapped pinned host memory the host can poll without synchronising.
+// Where kernels report a failure: the step's own word (later kernels of the
+// same step skip their work when it is set), the handle's word (what the host
+// reports), and a flag in mapped pinned host memory the host polls without
+// synchronising.
 struct ErrSink {
+  uint32_t* step;
   uint32_t* dev;
   volatile uint32_t* host;
 };
 
 __device__ __forceinline__ void raise_error(const ErrSink& e, uint32_t code) {
+  atomicOr(e.step, code);
   atomicOr(e.dev, code);
   *e.host = 1u;
 }
@@ -122,6 +126,7 @@ struct StepScratch {
   int32_t* keep;           // [M] message weights f
   int32_t* kept_list;      // [M] indices of kept messages, in pop order
   int32_t* n_kept;         // [1]
+  uint32_t* step_err;      // [1] failures of this step
 };
 
 // Accumulated statistics (device).

@@ -131,7 +131,7 @@ extern "C" gba_status gba_sort_ids_static(const int64_t* ids, int64_t n, int64_t
   sc.hist = reinterpret_cast<uint32_t*>(base + kOffHist);
   sc.tile_counter = reinterpret_cast<uint32_t*>(base + kOffTiles);
   uint32_t* err_words = reinterpret_cast<uint32_t*>(base + kOffErr);
-  ErrSink err{err_words, err_words + 1};
+  ErrSink err{err_words, err_words, err_words + 1};
 
   uint64_t kmax = (uint64_t)rows - 1;
   int bits = 1;

@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 4 : (EPL == 2 ? 3 : 1)
   __shared__ float s_pend_den[SEG_WARPS][QR];
   extern __shared__ __align__(16) float s_dyn[];  // staged rows, then the queue
 
-  if (ld_volatile_u32(err.dev) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  if (ld_volatile_u32(err.step) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
   const int M = a.M;
   const uint32_t* off_g = a.msg_off + (size_t)tb.t * (M + 1);
   const float* const* rows_g = a.rows_ptr + (size_t)tb.t * M;
@@ -581,7 +581,7 @@ __global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 3 : 2)
   __shared__ float s_pend_den[SEG_WARPS][QCAP];
   extern __shared__ __align__(16) float s_dyn[];  // staged rows, then the queue
 
-  if (ld_volatile_u32(err.dev) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  if (ld_volatile_u32(err.step) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
   const int M = a.M;
   const uint32_t* off_g = a.msg_off + (size_t)tb.t * (M + 1);
   const float* const* rows_g = a.rows_ptr + (size_t)tb.t * M;
@@ -841,7 +841,7 @@ constexpr int FIX_MAX_PER_LANE = 8;  // dims up to 256
 __global__ void __launch_bounds__(256)
     k_segsum_fixup(StepArgs a, SegTable tb, int64_t n_warps, SegRecords rec, DevStats* st,
                    uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err) {
-  if (ld_volatile_u32(err.dev) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  if (ld_volatile_u32(err.step) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t w = (int64_t)blockIdx.x * 8 + warp;
   if (w >= n_warps) return;

@@ -124,6 +124,7 @@ __global__ void __launch_bounds__(256) k_message_weights(StepArgs a, StepScratch
   const int tid = threadIdx.x;
   for (int i = tid; i < n_hist_words; i += blockDim.x) sc.hist[i] = 0u;
   if (tid < MAX_PASSES) sc.tile_counter[tid] = 0u;
+  if (tid == 0) *sc.step_err = 0u;
   if (tid >= 32) return;
   const int lane = tid;
   int kept = 0;
@@ -203,7 +204,7 @@ __global__ void __launch_bounds__(SORT_THREADS)
 
   // An id range error was latched before this launch (by the histogram):
   // every tile of every pass skips, consistently.
-  if (ld_volatile_u32(err.dev) & ERR_ID_RANGE) return;
+  if (ld_volatile_u32(err.step) & ERR_ID_RANGE) return;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) s_tile = atomicAdd(sc.tile_counter + pass, 1u);
@@ -297,7 +298,7 @@ __global__ void __launch_bounds__(SORT_THREADS)
       if (done) break;
       j -= used;
       if (j < 0) break;  // cannot happen: tile 0 publishes an inclusive prefix
-      if (used == 0 && ((ld_volatile_u32(err.dev) & ERR_TIMEOUT) ||
+      if (used == 0 && ((ld_volatile_u32(err.step) & ERR_TIMEOUT) ||
                         (int64_t)(globaltimer_ns() - t0) > wait_ns)) {
         raise_error(err, ERR_TIMEOUT);
         break;

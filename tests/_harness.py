@@ -22,7 +22,7 @@ def opt_desc(o: W.OptCfg):
     return B.opt_desc(o.kind, o.lr, o.init_acc, o.beta1, o.beta2, o.eps)
 
 
-def make_gpu(cfg: W.WorkloadCfg, max_buf=None, seed=None, debug=True, rule=None):
+def make_gpu(cfg: W.WorkloadCfg, max_buf=None, seed=None, debug=True, rule=None, overlap=False):
     tables = [(tb.rows, tb.dim, tb.id_mode, cfg.max_ids_per_msg(t), opt_desc(tb.opt))
               for t, tb in enumerate(cfg.tables)]
     rule = rule or dict(iota=cfg.iota)
@@ -30,6 +30,8 @@ def make_gpu(cfg: W.WorkloadCfg, max_buf=None, seed=None, debug=True, rule=None)
               seed=cfg.seed if seed is None else seed, **rule)
     if debug:
         g.set_debug(True)
+    if overlap:
+        g.set_overlap(True)
     return g
 
 
@@ -149,10 +151,10 @@ def accumulate_stats(acc: dict, step: dict, orc=None):
 
 def run_parity(cfg: W.WorkloadCfg, steps: int, tol: float, by_ref=False, check_every=1,
                track_rows=None, track_dense=None, max_buf=None, rule=None, device="cuda",
-               messages=None):
+               messages=None, overlap=False):
     """Feed the same stream to both sides for `steps` global steps and compare."""
     full = track_rows is None
-    g = make_gpu(cfg, max_buf=max_buf, rule=rule)
+    g = make_gpu(cfg, max_buf=max_buf, rule=rule, overlap=overlap)
     orc = make_oracle(cfg, track_rows, track_dense, rule=rule)
     stats = {}
     worst = {}
@@ -193,11 +195,11 @@ def rows_of_gpu(tb, ids: torch.Tensor) -> torch.Tensor:
 
 
 def run_fullsize(cfg: W.WorkloadCfg, steps: int, tol: float, n_hot=150, n_rand=1500,
-                 n_dense=20000, seed=0):
+                 n_dense=20000, seed=0, overlap=True):
     """Full-size workload in the benchmark's launch configuration (messages
     pushed by reference), checked against the oracle on a sample of rows (hot
     and random rows touched by the first step) and of dense parameters."""
-    g = make_gpu(cfg, debug=False)
+    g = make_gpu(cfg, debug=False, overlap=overlap)
     gen = torch.Generator().manual_seed(seed)
     first = W.generate_step(cfg, 0, "cuda")
     track = []

@@ -28,9 +28,12 @@ def test_reduced_configs_few_steps(n):
 
 
 @pytest.mark.parametrize("n", [2, 3, 5])
-def test_reduced_configs_by_reference(n):
+@pytest.mark.parametrize("overlap", [False, True])
+def test_reduced_configs_by_reference(n, overlap):
+    """Messages pushed by reference; with overlap on, consecutive steps run
+    concurrently (the next step's sort during this step's row update)."""
     cfg = W.reduced(n)
-    H.run_parity(cfg, steps=3, tol=H.TOL_ONE_STEP, by_ref=True)
+    H.run_parity(cfg, steps=4, tol=H.TOL_ONE_STEP, by_ref=True, overlap=overlap)
 
 
 @pytest.mark.parametrize("n", [1, 2, 3, 4, 5])
@@ -38,7 +41,8 @@ def test_hundred_steps(n):
     cfg = W.reduced(n)
     if n == 3:  # multi-hot: keep the oracle's run short, fewer ids per message
         cfg = W.replace(cfg, B=6)
-    H.run_parity(cfg, steps=100, tol=H.TOL_MANY_STEPS, check_every=25, by_ref=True)
+    H.run_parity(cfg, steps=100, tol=H.TOL_MANY_STEPS, check_every=25, by_ref=True,
+                 overlap=(n % 2 == 1))
 
 
 def test_config1_full_twenty_steps():
