@@ -500,57 +500,76 @@ __device__ __forceinline__ void copy_row_smem(float* dst, const float* src, int 
   }
 }
 
-// Lane = row: applies queued rows [0, npend), 32 at a time.
+// Applies queued rows [0, npend).  When d is a multiple of 4, L = d/4 lanes
+// share a row, each lane one 16-byte piece (so a row is one coalesced access)
+// and the warp updates 32/L rows at a time; otherwise one lane per row.
 __device__ __noinline__ void apply_queue(const StepArgs& a, const SegTable& tb, int lane,
                                          const float* pend, const uint32_t* pend_x,
                                          const float* pend_den, int qs, int& npend) {
   const int d = tb.d;
   const bool adam = tb.opt.kind == 1;
   __syncwarp();
-  for (int b0 = 0; b0 < npend; b0 += 32) {
-    const int i = b0 + lane;
-    if (i < npend) {
-      const uint32_t x = pend_x[i];
-      const float den = pend_den[i];
-      const float* g = pend + (size_t)i * qs;
-      float* w = tb.w + (size_t)x * d;
-      float* s0 = tb.s0 + (size_t)x * d;
-      float* s1 = adam ? tb.s1 + (size_t)x * d : nullptr;
-      if ((d & 3) == 0) {
-        constexpr int U = 2;  // 16-byte pieces in flight per lane and array
-        for (int c0 = 0; c0 < d; c0 += 4 * U) {
-          float4 wv[U], av[U], bv[U], gv[U];
+  if ((d & 3) == 0) {
+    const int L = d >> 2;                 // lanes per row (d <= 64: L <= 16)
+    const int G = 32 / L;                 // rows per pass
+    const int g = lane / L, l = lane - g * L;
+    const bool on = g < G;                // lanes past G * L idle (L not a power of two)
+    for (int i0 = 0; i0 < npend; i0 += 2 * G) {
+      // two rows per lane group in flight
+      const int ia = i0 + g, ib = i0 + G + g;
+      const bool va = on && ia < npend, vb = on && ib < npend;
+      float4 wa, aa, ba, wb, ab, bb;
+      uint32_t xa = 0u, xb = 0u;
+      if (va) {
+        xa = pend_x[ia];
+        const size_t r = (size_t)xa * d + 4 * l;
+        wa = *reinterpret_cast<const float4*>(tb.w + r);
+        aa = *reinterpret_cast<const float4*>(tb.s0 + r);
+        if (adam) ba = *reinterpret_cast<const float4*>(tb.s1 + r);
+      }
+      if (vb) {
+        xb = pend_x[ib];
+        const size_t r = (size_t)xb * d + 4 * l;
+        wb = *reinterpret_cast<const float4*>(tb.w + r);
+        ab = *reinterpret_cast<const float4*>(tb.s0 + r);
+        if (adam) bb = *reinterpret_cast<const float4*>(tb.s1 + r);
+      }
 #pragma unroll
-          for (int u = 0; u < U; ++u) {
-            const int c = c0 + 4 * u;
-            if (c < d) {
-              wv[u] = *reinterpret_cast<const float4*>(w + c);
-              av[u] = *reinterpret_cast<const float4*>(s0 + c);
-              if (adam) bv[u] = *reinterpret_cast<const float4*>(s1 + c);
-              gv[u] = *reinterpret_cast<const float4*>(g + c);
-            }
-          }
+      for (int h = 0; h < 2; ++h) {
+        const bool v = h == 0 ? va : vb;
+        if (!v) continue;
+        const int i = h == 0 ? ia : ib;
+        const uint32_t x = h == 0 ? xa : xb;
+        float4 wv = h == 0 ? wa : wb, av = h == 0 ? aa : ab, bv = h == 0 ? ba : bb;
+        const float4 gv = *reinterpret_cast<const float4*>(pend + (size_t)i * qs + 4 * l);
+        const float den = pend_den[i];
+        float* wp = &wv.x;
+        float* ap = &av.x;
+        float* bp = &bv.x;
+        const float* gp = &gv.x;
 #pragma unroll
-          for (int u = 0; u < U; ++u) {
-            const int c = c0 + 4 * u;
-            if (c < d) {
-              float* wp = &wv[u].x;
-              float* ap = &av[u].x;
-              float* bp = &bv[u].x;
-              const float* gp = &gv[u].x;
-#pragma unroll
-              for (int k = 0; k < 4; ++k) {
-                float bk = adam ? bp[k] : 0.f;
-                opt_update(tb.opt, wp[k], ap[k], bk, den == 1.0f ? gp[k] : __fdiv_rn(gp[k], den));
-                bp[k] = bk;
-              }
-              *reinterpret_cast<float4*>(w + c) = wv[u];
-              *reinterpret_cast<float4*>(s0 + c) = av[u];
-              if (adam) *reinterpret_cast<float4*>(s1 + c) = bv[u];
-            }
-          }
+        for (int k = 0; k < 4; ++k) {
+          float bk = adam ? bp[k] : 0.f;
+          opt_update(tb.opt, wp[k], ap[k], bk, den == 1.0f ? gp[k] : __fdiv_rn(gp[k], den));
+          bp[k] = bk;
         }
-      } else {
+        const size_t r = (size_t)x * d + 4 * l;
+        *reinterpret_cast<float4*>(tb.w + r) = wv;
+        *reinterpret_cast<float4*>(tb.s0 + r) = av;
+        if (adam) *reinterpret_cast<float4*>(tb.s1 + r) = bv;
+        if (l == 0) tb.ver[x] = (int32_t)(a.k + 1);
+      }
+    }
+  } else {
+    for (int b0 = 0; b0 < npend; b0 += 32) {
+      const int i = b0 + lane;
+      if (i < npend) {
+        const uint32_t x = pend_x[i];
+        const float den = pend_den[i];
+        const float* g = pend + (size_t)i * qs;
+        float* w = tb.w + (size_t)x * d;
+        float* s0 = tb.s0 + (size_t)x * d;
+        float* s1 = adam ? tb.s1 + (size_t)x * d : nullptr;
         for (int c = 0; c < d; ++c) {
           float wk = w[c], ak = s0[c], bk = adam ? s1[c] : 0.f;
           opt_update(tb.opt, wk, ak, bk, den == 1.0f ? g[c] : __fdiv_rn(g[c], den));
@@ -558,8 +577,8 @@ __device__ __noinline__ void apply_queue(const StepArgs& a, const SegTable& tb, 
           s0[c] = ak;
           if (adam) s1[c] = bk;
         }
+        tb.ver[x] = (int32_t)(a.k + 1);
       }
-      tb.ver[x] = (int32_t)(a.k + 1);
     }
   }
   npend = 0;
@@ -672,6 +691,7 @@ __global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 3 : 2)
     // ---- lane j: metadata of position rb + j; its gradient row is staged if kept
     uint32_t key = 0xFFFFFFFFu, m = 0xFFFFFFFEu, stale = 0u;
     bool keep = false;
+    const float* my_row = nullptr;
     if (valid) {
       key = keys[rb + lane];
       const uint32_t o_t = (uint32_t)((int64_t)vals[rb + lane] - nbase);
@@ -688,7 +708,7 @@ __global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 3 : 2)
         const uint64_t sl = diff > 0 ? (uint64_t)diff : 0ull;
         keep = sl <= (uint64_t)(int64_t)a.iota;
         stale = (uint32_t)(sl > 0xFFFFFFFFull ? 0xFFFFFFFFull : sl);
-        if (keep) stage_row(stage + lane * SS, rowp, d);
+        my_row = rowp;
       }
     }
     uint32_t pk = __shfl_up_sync(0xffffffffu, key, 1);
@@ -710,6 +730,24 @@ __global__ void __launch_bounds__(SEG_THREADS, EPL == 1 ? 3 : 2)
     const uint32_t Km = __ballot_sync(0xffffffffu, keep);
     const uint32_t Nm = __ballot_sync(0xffffffffu, newmsg);
     const uint32_t Vm = __ballot_sync(0xffffffffu, valid);
+    // ---- stage the kept gradient rows: L = d/4 lanes per row, one 16-byte
+    // piece each (a row is one coalesced access); 4-byte copies otherwise
+    if ((d & 3) == 0) {
+      const int L = d >> 2, G = 32 / L;
+      const int g = lane / L, l = lane - g * L;
+      for (int j0 = 0; j0 < n_round; j0 += G) {
+        const int j = j0 + g;
+        const float* src = (const float*)__shfl_sync(0xffffffffu, (unsigned long long)my_row,
+                                                     j < 32 ? j : 31);
+        if (g < G && j < n_round && ((Km >> j) & 1u))
+          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                           smem_u32(stage + j * SS + 4 * l)),
+                       "l"(src + 4 * l)
+                       : "memory");
+      }
+    } else if (keep) {
+      stage_row(stage + lane * SS, my_row, d);
+    }
     const uint32_t Bm = (Hm | 1u) & Vm;  // segment starts (position 0 always starts one)
     const int last_start = 31 - __clz(Bm);
     const bool starts = (Bm >> lane) & 1u;
