@@ -61,10 +61,10 @@ def alg_bytes(cfg, st_delta, steps):
     m_kept = st_delta["msgs_kept"] / steps
     b = {
         "sort": 8.0 * occ,
-        "segsum": 4.0 * d * occ_kept + 2 * s_opt_rows * 4.0 * d * u_app + 8.0 * u_app,
+        "rows": 4.0 * d * occ_kept + 2 * s_opt_rows * 4.0 * d * u_app + 8.0 * u_app,
         "dense": 4.0 * cfg.D * m_kept + 2 * s_opt_dense * 4.0 * cfg.D,
     }
-    b["total"] = b["sort"] + b["segsum"] + b["dense"]
+    b["total"] = b["sort"] + b["rows"] + b["dense"]
     return b, dict(occ=occ, occ_kept=occ_kept, u_applied=u_app, m_kept=m_kept,
                    u_touched=st_delta["rows_touched"] / steps)
 
@@ -121,7 +121,7 @@ def source_sha(files):
 
 
 KERNEL_SOURCES = {
-    "segsum": ["paper_2205_11048_gb300/csrc/gba_segsum.cu", "paper_2205_11048_gb300/csrc/gba_internal.cuh"],
+    "rows": ["paper_2205_11048_gb300/csrc/gba_rows.cu", "paper_2205_11048_gb300/csrc/gba_internal.cuh"],
     "dense": ["paper_2205_11048_gb300/csrc/gba_dense.cu", "paper_2205_11048_gb300/csrc/gba_internal.cuh"],
     "sort": ["paper_2205_11048_gb300/csrc/gba_sort.cu", "paper_2205_11048_gb300/csrc/gba_internal.cuh"],
 }
@@ -336,10 +336,13 @@ def run_gba(args):
     # roofline of the dominant kernel class: the one that must move the most
     # algorithmic bytes (its time is measured live, concurrent steps included)
     bytes_, per = alg_bytes(cfg, delta, args.steps)
-    classes = {"segsum": kt["segsum"][1] + kt["fixup"][1], "dense": kt["dense"][1],
-               "sort": kt["sort_hist"][1] + kt["sort_pass"][1]}
-    dom = max(("segsum", "dense", "sort"), key=lambda c: bytes_[c])
-    n_launch = {"segsum": kt["segsum"][0], "dense": kt["dense"][0], "sort": kt["sort_pass"][0]}
+    # the row path is three kernels per table (segment reduction, rows that
+    # cross windows, row update): its bytes are divided by their summed time
+    classes = {"rows": kt["seg_reduce"][1] + kt["seg_cross"][1] + kt["row_update"][1],
+               "dense": kt["dense"][1], "sort": kt["sort_hist"][1] + kt["sort_pass"][1]}
+    dom = max(("rows", "dense", "sort"), key=lambda c: bytes_[c])
+    n_launch = {"rows": kt["seg_reduce"][0] + kt["seg_cross"][0] + kt["row_update"][0],
+                "dense": kt["dense"][0], "sort": kt["sort_hist"][0] + kt["sort_pass"][0]}
     launches_per_step = max(1, n_launch[dom] // args.steps)
     dur_ms = classes[dom] / args.steps  # one step's launches of that class
     peak, peak_kind = peaks()

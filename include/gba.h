@@ -107,15 +107,18 @@ typedef struct {
 } gba_stats_t;
 
 /* Per kernel class: launches and device time summed since timing was enabled. */
-typedef struct {
-  int64_t launches[8];
-  double ms[8];
-} gba_kernel_times_t;
-/* indices into gba_kernel_times_t */
+/* indices into gba_kernel_times_t: K1 message weights; K2 sort (digit
+ * histograms, one onesweep pass per key byte); K3 segment reduction, rows that
+ * cross reduction windows, K4 row update; K5 dense update; table init. */
 enum {
-  GBA_K_WEIGHTS = 0, GBA_K_SORT_HIST = 1, GBA_K_SORT_PASS = 2, GBA_K_SEGSUM = 3,
-  GBA_K_FIXUP = 4, GBA_K_DENSE = 5, GBA_K_INIT = 6, GBA_K_OTHER = 7
+  GBA_K_WEIGHTS = 0, GBA_K_SORT_HIST = 1, GBA_K_SORT_PASS = 2, GBA_K_SEG_REDUCE = 3,
+  GBA_K_SEG_CROSS = 4, GBA_K_ROW_UPDATE = 5, GBA_K_DENSE = 6, GBA_K_INIT = 7,
+  GBA_K_OTHER = 8, GBA_K_COUNT = 9
 };
+typedef struct {
+  int64_t launches[GBA_K_COUNT];
+  double ms[GBA_K_COUNT];
+} gba_kernel_times_t;
 
 /*
  * gba_create - allocate the parameter-server state on the current device.

@@ -30,7 +30,8 @@ STATUS_NAMES = {0: "GBA_OK", -1: "GBA_E_ARG", -2: "GBA_E_ID_RANGE", -3: "GBA_E_O
 ADAGRAD, ADAM = 0, 1
 DIRECT, MODULO = 0, 1
 INT32_MAX = 2**31 - 1
-KERNEL_NAMES = ["weights", "sort_hist", "sort_pass", "segsum", "fixup", "dense", "init", "other"]
+KERNEL_NAMES = ["weights", "sort_hist", "sort_pass", "seg_reduce", "seg_cross", "row_update",
+                "dense", "init", "other"]
 
 
 class GBAError(RuntimeError):
@@ -70,7 +71,8 @@ class gba_stats_t(ctypes.Structure):
 
 
 class gba_kernel_times_t(ctypes.Structure):
-    _fields_ = [("launches", ctypes.c_int64 * 8), ("ms", ctypes.c_double * 8)]
+    _fields_ = [("launches", ctypes.c_int64 * len(KERNEL_NAMES)),
+                ("ms", ctypes.c_double * len(KERNEL_NAMES))]
 
 
 _P = ctypes.c_void_p
@@ -320,7 +322,7 @@ class GBA:
     def kernel_times(self):
         kt = gba_kernel_times_t()
         check(self.L.gba_kernel_times(self.h, ctypes.byref(kt)), self.h)
-        return {KERNEL_NAMES[i]: (int(kt.launches[i]), float(kt.ms[i])) for i in range(8)}
+        return {KERNEL_NAMES[i]: (int(kt.launches[i]), float(kt.ms[i])) for i in range(len(KERNEL_NAMES))}
 
     def set_wait_limit(self, ns):
         check(self.L.gba_debug_set_wait_limit(self.h, int(ns)), self.h)

@@ -132,8 +132,16 @@ struct gba_handle {
   int64_t dbg_cap = 0;
   char* d_step_scratch[SLOTS] = {};
   StepScratch sc[SLOTS] = {};
-  SegRecords rec{};
-  int64_t rec_warps = 0;
+  // segment-sum and row-update buffers (apply stream only), grown with n_cap
+  RowDesc* d_desc = nullptr;
+  float* d_compact = nullptr;
+  float* d_rec_hi = nullptr;
+  float* d_rec_lo = nullptr;
+  uint32_t* d_rec_meta = nullptr;
+  unsigned long long* d_seg_status = nullptr;
+  uint32_t* d_seg_total = nullptr;
+  uint32_t* d_cross_list = nullptr;
+  int64_t seg_win_cap = 0;
   int d_max = 1;
 
   uint32_t* d_err = nullptr;
@@ -284,9 +292,14 @@ void free_all(gba_handle* h) {
   }
   cudaFree(h->d_dbg_count);
   cudaFree(h->d_dbg_kept);
-  cudaFree(h->rec.hi);
-  cudaFree(h->rec.lo);
-  cudaFree(h->rec.meta);
+  cudaFree(h->d_desc);
+  cudaFree(h->d_compact);
+  cudaFree(h->d_rec_hi);
+  cudaFree(h->d_rec_lo);
+  cudaFree(h->d_rec_meta);
+  cudaFree(h->d_seg_status);
+  cudaFree(h->d_seg_total);
+  cudaFree(h->d_cross_list);
   cudaFree(h->d_err);
   if (h->h_err) cudaFreeHost(h->h_err);
   cudaFree(h->d_stats);
@@ -369,6 +382,27 @@ gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
     }
     h->n_cap = cap;
     h->status_tiles = tiles;
+    // segment buffers: one list entry (and compact row) per possible row head,
+    // records and look-back words per window
+    const int64_t cs = (h->d_max + 3) / 4 * 4;
+    const int64_t wins = seg_window_bound(cap, h->num_sms);
+    for (void* p : {(void*)h->d_desc, (void*)h->d_compact, (void*)h->d_rec_hi, (void*)h->d_rec_lo,
+                    (void*)h->d_rec_meta, (void*)h->d_seg_status, (void*)h->d_cross_list})
+      cudaFree(p);
+    h->d_cross_list = nullptr;
+    h->d_desc = nullptr;
+    h->d_compact = h->d_rec_hi = h->d_rec_lo = nullptr;
+    h->d_rec_meta = nullptr;
+    h->d_seg_status = nullptr;
+    GBA_CUDA(h, cudaMalloc(&h->d_desc, cap * sizeof(RowDesc)));
+    GBA_CUDA(h, cudaMalloc(&h->d_compact, (size_t)cap * cs * sizeof(float)));
+    GBA_CUDA(h, cudaMalloc(&h->d_rec_hi, (size_t)wins * 2 * h->d_max * sizeof(float)));
+    GBA_CUDA(h, cudaMalloc(&h->d_rec_lo, (size_t)wins * 2 * h->d_max * sizeof(float)));
+    GBA_CUDA(h, cudaMalloc(&h->d_rec_meta, (size_t)wins * 2 * REC_META * sizeof(uint32_t)));
+    GBA_CUDA(h, cudaMalloc(&h->d_seg_status, (size_t)wins * sizeof(unsigned long long)));
+    GBA_CUDA(h, cudaMalloc(&h->d_cross_list, (size_t)wins * sizeof(uint32_t)));
+    GBA_CUDA(h, cudaMemset(h->d_seg_status, 0, (size_t)wins * sizeof(unsigned long long)));
+    h->seg_win_cap = wins;
   }
   if (h->debug && N > h->dbg_cap) {
     sync_all(h);
@@ -621,7 +655,8 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   {
     const size_t M = (size_t)max_buffered_msgs;
     const size_t bytes = align16(MAX_PASSES * 256 * 4) + align16(MAX_PASSES * 4) +
-                         align16(M * 4) + align16(M * 4) + align16(4) + align16(4);
+                         align16(M * 4) + align16(M * 4) + align16(4) + align16(4) +
+                         align16((size_t)std::max(h->T, 1) * 8);
     for (int b = 0; b < SLOTS; ++b) {
       if (!dev_alloc((void**)&h->d_step_scratch[b], bytes)) return fail(GBA_E_OOM);
       if (cudaMemset(h->d_step_scratch[b], 0, bytes) != cudaSuccess) return fail(GBA_E_CUDA);
@@ -638,15 +673,11 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
       sc.n_kept = (int32_t*)p;
       p += align16(4);
       sc.step_err = (uint32_t*)p;
+      p += align16(4);
+      sc.seg_ticket = (uint32_t*)p;
     }
   }
-  {
-    h->rec_warps = (int64_t)h->num_sms * 64 + 64;
-    const size_t nf = (size_t)h->rec_warps * 2 * h->d_max;
-    if (!dev_alloc((void**)&h->rec.hi, nf * 4) || !dev_alloc((void**)&h->rec.lo, nf * 4) ||
-        !dev_alloc((void**)&h->rec.meta, (size_t)h->rec_warps * 2 * 6 * 4))
-      return fail(GBA_E_OOM);
-  }
+  if (!dev_alloc((void**)&h->d_seg_total, 16)) return fail(GBA_E_OOM);
   if (!dev_alloc((void**)&h->d_err, 4) || !dev_alloc((void**)&h->d_stats, sizeof(DevStats)))
     return fail(GBA_E_OOM);
   if (cudaHostAlloc((void**)&h->h_err, 4, cudaHostAllocMapped) != cudaSuccess)
@@ -861,16 +892,34 @@ int32_t gba_try_apply(gba_handle* h) {
       tb.opt = make_opt_step(ts.desc.opt, p1, p2);
       uint32_t* dc = h->debug ? h->d_dbg_count : nullptr;
       uint32_t* dk = h->debug ? h->d_dbg_kept : nullptr;
-      int64_t n_warps = 0;
+      if (++h->epoch == 0u) h->epoch = 1u;
+      SegOut so{};
+      so.desc = h->d_desc;
+      so.compact = h->d_compact;
+      so.cs = (tb.d + 3) / 4 * 4;
+      so.rec_stride = h->d_max;
+      so.rec_hi = h->d_rec_hi;
+      so.rec_lo = h->d_rec_lo;
+      so.rec_meta = h->d_rec_meta;
+      so.status = h->d_seg_status;
+      so.epoch = h->epoch;
+      so.ticket = sc.seg_ticket + 2 * t;
+      so.cross_count = sc.seg_ticket + 2 * t + 1;
+      so.cross_list = h->d_cross_list;
+      so.total = h->d_seg_total;
+      int64_t n_win = 0;
       {
-        Timed tm(h, GBA_K_SEGSUM, h->applys);
-        n_warps = launch_segsum(a, tb, h->d_keys[b][final_buf], h->d_vals[b][final_buf],
-                                h->rec, h->rec_warps, h->d_stats, dc, dk, sink, h->num_sms,
-                                h->applys);
+        Timed tm(h, GBA_K_SEG_REDUCE, h->applys);
+        n_win = launch_seg_reduce(a, tb, so, h->d_keys[b][final_buf], h->d_vals[b][final_buf],
+                                  h->d_stats, dc, dk, sink, h->num_sms, h->wait_ns, h->applys);
       }
       {
-        Timed tm(h, GBA_K_FIXUP, h->applys);
-        launch_fixup(a, tb, n_warps, h->rec, h->d_stats, dc, dk, sink, h->applys);
+        Timed tm(h, GBA_K_SEG_CROSS, h->applys);
+        launch_seg_cross(a, tb, so, n_win, dc, dk, sink, h->applys);
+      }
+      {
+        Timed tm(h, GBA_K_ROW_UPDATE, h->applys);
+        launch_row_update(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
       }
     }
   }

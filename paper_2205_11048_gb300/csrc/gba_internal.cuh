@@ -33,6 +33,57 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// ---- mbarriers and 1-D bulk async copies (shared memory, this CTA) ----------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0u;
+}
+
+// Bounded wait for the phase with the given parity; false if it gave up.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if ((int64_t)(globaltimer_ns() - t0) > limit_ns) return false;
+  }
+  return true;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes,
+                                         uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
 // ---- per-table static description (device copy) ----------------------------
 struct TableInfo {
   int64_t V;
@@ -127,6 +178,7 @@ struct StepScratch {
   int32_t* kept_list;      // [M] indices of kept messages, in pop order
   int32_t* n_kept;         // [1]
   uint32_t* step_err;      // [1] failures of this step
+  uint32_t* seg_ticket;    // [T][2] window tickets and crossing-row counts of the segment kernels
 };
 
 // Accumulated statistics (device).
@@ -179,25 +231,50 @@ struct SegTable {
   OptStep opt;
 };
 
-// Partial sums of rows that cross warp ranges: per warp range, slot 0 is the
-// part of a row that began in an earlier range, slot 1 the part of a row that
-// begins in this range and continues into the next.
-struct SegRecords {
-  float* hi;       // [W][2][d_max] compensated partial sums
-  float* lo;       // [W][2][d_max]
-  uint32_t* meta;  // [W][2][6]  type, x, c_all, c_kept, k_occ, head_pos
+// One row of the step's compact update list: where its aggregated gradient
+// is (a message's gradient row when one occurrence was kept, else the compact
+// buffer), the row, and the denominator of its weighted sum (0: no update).
+struct RowDesc {
+  const float* src;
+  uint32_t x;
+  float den;
 };
 
-// Launches the segment-sum + row update over table tb's range of the sorted
-// array; returns the number of warp ranges (for the fixup launch).
-int64_t launch_segsum(const StepArgs& a, const SegTable& tb, const uint32_t* keys,
-                      const uint32_t* vals, SegRecords rec, int64_t max_warps, DevStats* stats,
-                      uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
-                      cudaStream_t s);
+constexpr int REC_META = 8;  // type, x, c_all, c_kept, k_occ, head_pos, u, unused
 
-void launch_fixup(const StepArgs& a, const SegTable& tb, int64_t n_warps, SegRecords rec,
-                  DevStats* stats, uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err,
-                  cudaStream_t s);
+// Buffers of the segment-sum and row-update kernels (one set, used in stream
+// order by the apply stream).
+struct SegOut {
+  RowDesc* desc;              // [U] the step's rows in sorted order
+  float* compact;             // [U][cs] sums of rows with two or more kept occurrences
+  int32_t cs;                 // compact row stride (floats, a multiple of 4)
+  int32_t rec_stride;         // floats per record
+  float* rec_hi;              // [windows][2][rec_stride] compensated partial sums
+  float* rec_lo;              // [windows][2][rec_stride]
+  uint32_t* rec_meta;         // [windows][2][REC_META]
+  unsigned long long* status; // [windows] look-back words
+  uint32_t epoch;             // tag of this launch's look-back words
+  uint32_t* ticket;           // window tickets (cleared by K1)
+  uint32_t* cross_count;      // rows that cross windows (cleared by K1)
+  uint32_t* cross_list;       // [windows] windows where such a row begins
+  uint32_t* total;            // U, written by the last window
+};
+
+// Upper bound on the windows of a table of N sorted positions.
+int64_t seg_window_bound(int64_t N, int num_sms);
+
+// Segment reduction over table tb's range of the sorted array; returns the
+// number of windows (for the cross-window kernel).
+int64_t launch_seg_reduce(const StepArgs& a, const SegTable& tb, const SegOut& so,
+                          const uint32_t* keys, const uint32_t* vals, DevStats* stats,
+                          uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
+                          int64_t wait_ns, cudaStream_t s);
+
+void launch_seg_cross(const StepArgs& a, const SegTable& tb, const SegOut& so, int64_t n_win,
+                      uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, cudaStream_t s);
+
+void launch_row_update(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
+                       ErrSink err, int num_sms, cudaStream_t s);
 
 struct DenseArgs {
   float* w;
