@@ -284,7 +284,7 @@ gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream);
  * cleared at the start of each call); calls whose work overlaps on the GPU race.
  */
 #define GBA_STATIC_SORT_MAX_IDS (1 << 20)
-#define GBA_STATIC_SORT_BYTES 8917104
+#define GBA_STATIC_SORT_BYTES 9441392
 gba_status gba_sort_ids_static(const int64_t* ids, int64_t n, int64_t rows, int32_t id_mode,
                                uint32_t* rows_out, uint32_t* order_out, void* cuda_stream);
 

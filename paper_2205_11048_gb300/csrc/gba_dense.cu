@@ -5,11 +5,13 @@
 // or Adam in place -- one pass over HBM: every kept gradient is read once, the
 // weights and optimizer state are read and written once.
 //
-// Each persistent CTA walks tiles of 1024 parameters.  A producer warp streams
+// Each persistent CTA walks an equal contiguous share of the parameters in
+// tiles of up to 1024.  A producer warp streams
 // the tile's slice of every kept message into a ring of shared-memory stages
 // with 1-D bulk async copies (cp.async.bulk, completion counted on an mbarrier
-// per stage); eight consumer warps sum the slices with compensated float
-// arithmetic, release each stage on an "empty" mbarrier, and finish the tile
+// per stage); eight consumer warps sum the slices with compensated (TwoSum)
+// float arithmetic, release each stage on an "empty" mbarrier, and finish the
+// tile
 // with the optimizer.  Every mbarrier wait is bounded in time; a wait that
 // gives up latches ERR_TIMEOUT, the CTA stops issuing copies, waits (bounded)
 // for the copies it already issued, and exits.
@@ -32,7 +34,8 @@ __global__ void __launch_bounds__(DENSE_THREADS)
   uint64_t* empty = full + STAGES;
   __shared__ int s_abort;
 
-  if (*(volatile uint32_t*)err.step & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  // block-uniform: another kernel may set the word while this block reads it
+  if (__syncthreads_or((*(volatile uint32_t*)err.step & (ERR_ID_RANGE | ERR_TIMEOUT)) != 0u)) return;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) {
@@ -47,16 +50,19 @@ __global__ void __launch_bounds__(DENSE_THREADS)
 
   const int n_kept = *sc.n_kept;
   const int64_t D4 = da.D & ~3ll;  // parameters streamed by bulk copies
-  const int64_t n_tiles = (D4 + DT - 1) / DT;
+  // This CTA's contiguous range of parameters (equal shares, multiples of 4
+  // so every copy stays 16-byte aligned), walked in tiles of up to DT.
+  const int64_t q4 = D4 / 4;
+  const int64_t r0 = 4 * (q4 * (int64_t)blockIdx.x / gridDim.x);
+  const int64_t r1 = 4 * (q4 * ((int64_t)blockIdx.x + 1) / gridDim.x);
 
   if (warp == CONSUMER_WARPS) {
     // ---- producer
     if (lane == 0) {
       uint32_t q = 0;
       bool ok = true;
-      for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        const int64_t start = tile * DT;
-        const uint32_t bytes = (uint32_t)((D4 - start < DT ? D4 - start : DT) * sizeof(float));
+      for (int64_t start = r0; start < r1 && ok; start += DT) {
+        const uint32_t bytes = (uint32_t)((r1 - start < DT ? r1 - start : DT) * sizeof(float));
         for (int j = 0; j < n_kept; ++j, ++q) {
           const int stage = (int)(q % STAGES);
           const uint32_t ph = (q / STAGES) & 1u;
@@ -85,9 +91,8 @@ __global__ void __launch_bounds__(DENSE_THREADS)
     const int c = tid;
     const float Mf = (float)da.M;
     uint32_t q = 0;
-    for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-      const int64_t start = tile * DT;
-      const int64_t n = D4 - start < DT ? D4 - start : DT;
+    for (int64_t start = r0; start < r1; start += DT) {
+      const int64_t n = r1 - start < DT ? r1 - start : DT;
       const bool mine = (int64_t)c * 4 < n;
       const int64_t e = start + (int64_t)c * 4;
       float4 w = make_float4(0.f, 0.f, 0.f, 0.f), s0 = w, s1 = w;
@@ -105,9 +110,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
         const uint32_t ph = (q / STAGES) & 1u;
         // Every lane waits (acquiring the copied bytes); the verdict is made
         // warp-uniform so the warp leaves the loop together.
-        bool ok = mbar_wait(full + stage, ph, wait_ns);
-        ok = __all_sync(0xffffffffu, ok) &&
-             __shfl_sync(0xffffffffu, *(volatile int*)&s_abort, 0) == 0;
+        const bool ok = __all_sync(0xffffffffu, mbar_wait(full + stage, ph, wait_ns));
         if (!ok) {
           if (lane == 0) {
             raise_error(err, ERR_TIMEOUT);
@@ -126,7 +129,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
         __syncwarp();
         if (lane == 0) mbar_arrive(empty + stage);
       }
-      if (aborted) break;
+      if (aborted || __shfl_sync(0xffffffffu, *(volatile int*)&s_abort, 0) != 0) break;
       if (mine) {
         float wv[4] = {w.x, w.y, w.z, w.w}, a0[4] = {s0.x, s0.y, s0.z, s0.w},
               a1[4] = {s1.x, s1.y, s1.z, s1.w};

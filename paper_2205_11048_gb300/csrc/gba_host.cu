@@ -141,6 +141,7 @@ struct gba_handle {
   unsigned long long* d_seg_status = nullptr;
   uint32_t* d_seg_total = nullptr;
   uint32_t* d_cross_list = nullptr;
+  uint32_t* d_cross_end = nullptr;
   int64_t seg_win_cap = 0;
   int d_max = 1;
 
@@ -300,6 +301,7 @@ void free_all(gba_handle* h) {
   cudaFree(h->d_seg_status);
   cudaFree(h->d_seg_total);
   cudaFree(h->d_cross_list);
+  cudaFree(h->d_cross_end);
   cudaFree(h->d_err);
   if (h->h_err) cudaFreeHost(h->h_err);
   cudaFree(h->d_stats);
@@ -387,9 +389,10 @@ gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
     const int64_t cs = (h->d_max + 3) / 4 * 4;
     const int64_t wins = seg_window_bound(cap, h->num_sms);
     for (void* p : {(void*)h->d_desc, (void*)h->d_compact, (void*)h->d_rec_hi, (void*)h->d_rec_lo,
-                    (void*)h->d_rec_meta, (void*)h->d_seg_status, (void*)h->d_cross_list})
+                    (void*)h->d_rec_meta, (void*)h->d_seg_status, (void*)h->d_cross_list,
+                    (void*)h->d_cross_end})
       cudaFree(p);
-    h->d_cross_list = nullptr;
+    h->d_cross_list = h->d_cross_end = nullptr;
     h->d_desc = nullptr;
     h->d_compact = h->d_rec_hi = h->d_rec_lo = nullptr;
     h->d_rec_meta = nullptr;
@@ -401,6 +404,7 @@ gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
     GBA_CUDA(h, cudaMalloc(&h->d_rec_meta, (size_t)wins * 2 * REC_META * sizeof(uint32_t)));
     GBA_CUDA(h, cudaMalloc(&h->d_seg_status, (size_t)wins * sizeof(unsigned long long)));
     GBA_CUDA(h, cudaMalloc(&h->d_cross_list, (size_t)wins * sizeof(uint32_t)));
+    GBA_CUDA(h, cudaMalloc(&h->d_cross_end, (size_t)cap * sizeof(uint32_t)));
     GBA_CUDA(h, cudaMemset(h->d_seg_status, 0, (size_t)wins * sizeof(unsigned long long)));
     h->seg_win_cap = wins;
   }
@@ -855,10 +859,11 @@ int32_t gba_try_apply(gba_handle* h) {
     {
       Timed tm(h, GBA_K_SORT_HIST, h->sorts);
       int grid = (int)std::min<int64_t>((N + 255) / 256, (int64_t)h->num_sms * 8);
-      launch_sort_histogram(a, h->passes, sc, sink, std::max(grid, 1), h->sorts);
+      // the first pass writes buffer 0, so its input keys go to buffer 1
+      launch_sort_histogram(a, h->passes, sc, h->d_keys[b][1], sink, std::max(grid, 1), h->sorts);
     }
     launch_dense_side();
-    const uint32_t* kin = nullptr;
+    const uint32_t* kin = h->d_keys[b][1];
     const uint32_t* vin = nullptr;
     for (int p = 0; p < h->passes; ++p) {
       const int ob = p & 1;
@@ -906,6 +911,7 @@ int32_t gba_try_apply(gba_handle* h) {
       so.ticket = sc.seg_ticket + 2 * t;
       so.cross_count = sc.seg_ticket + 2 * t + 1;
       so.cross_list = h->d_cross_list;
+      so.cross_end = h->d_cross_end;
       so.total = h->d_seg_total;
       int64_t n_win = 0;
       {

@@ -53,14 +53,16 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
+// Waits for the phase with the given parity to complete; the thread may be
+// suspended in the instruction for up to the hinted time instead of spinning.
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_addr(bar)), "r"(parity)
+      : "r"(smem_addr(bar)), "r"(parity), "r"(100000u)
       : "memory");
   return ok != 0u;
 }
@@ -207,8 +209,13 @@ __device__ __forceinline__ int message_of(const uint32_t* off, int M, uint32_t x
 void launch_weights(const StepArgs& a, StepScratch sc, DevStats* stats, int n_hist_words,
                     cudaStream_t s);
 
-void launch_sort_histogram(const StepArgs& a, int passes, StepScratch sc, ErrSink err, int grid,
-                           cudaStream_t s);
+// Keys per onesweep tile (also sizes the look-back words of the static sort).
+constexpr int SORT_TILE_KEYS = 2048;
+
+// Digit histograms of every pass; writes each occurrence's key to keys0 (the
+// first onesweep pass's input).
+void launch_sort_histogram(const StepArgs& a, int passes, StepScratch sc, uint32_t* keys0,
+                           ErrSink err, int grid, cudaStream_t s);
 
 void launch_onesweep(const StepArgs& a, bool first, int pass, const uint32_t* keys_in,
                      const uint32_t* vals_in, uint32_t* keys_out, uint32_t* vals_out,
@@ -257,6 +264,7 @@ struct SegOut {
   uint32_t* ticket;           // window tickets (cleared by K1)
   uint32_t* cross_count;      // rows that cross windows (cleared by K1)
   uint32_t* cross_list;       // [windows] windows where such a row begins
+  uint32_t* cross_end;        // [U] window where a crossing row ends, by list index
   uint32_t* total;            // U, written by the last window
 };
 

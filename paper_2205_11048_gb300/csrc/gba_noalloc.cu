@@ -29,7 +29,7 @@ namespace gba {
 namespace {
 
 constexpr int64_t kMaxIds = GBA_STATIC_SORT_MAX_IDS;
-constexpr int64_t kTile = 4096;  // keys per onesweep tile
+constexpr int64_t kTile = SORT_TILE_KEYS;  // keys per onesweep tile
 constexpr int64_t kMaxTiles = (kMaxIds + kTile - 1) / kTile;
 constexpr int kMaxDevices = 64;
 
@@ -140,14 +140,15 @@ extern "C" gba_status gba_sort_ids_static(const int64_t* ids, int64_t n, int64_t
 
   int grid = (int)((n + 255) / 256);
   if (grid > 152 * 8) grid = 152 * 8;
-  launch_sort_histogram(a, passes, sc, err, grid, s);
-
   // Ping-pong between the scratch pair and the caller's outputs so that the
-  // last pass lands in the outputs.
+  // last pass lands in the outputs; the first pass reads the keys the
+  // histogram kernel wrote into the buffer that pass does not write.
   uint32_t* tmp_k = reinterpret_cast<uint32_t*>(base + kOffKeys);
   uint32_t* tmp_v = reinterpret_cast<uint32_t*>(base + kOffVals);
   unsigned long long* status = reinterpret_cast<unsigned long long*>(base + kOffStatus);
-  const uint32_t* kin = nullptr;
+  uint32_t* keys0 = ((passes - 1) % 2) == 0 ? tmp_k : rows_out;
+  launch_sort_histogram(a, passes, sc, keys0, err, grid, s);
+  const uint32_t* kin = keys0;
   const uint32_t* vin = nullptr;
   for (int p = 0; p < passes; ++p) {
     const bool to_out = ((passes - 1 - p) % 2) == 0;

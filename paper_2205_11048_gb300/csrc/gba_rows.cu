@@ -13,8 +13,9 @@
 //                 look-back over the windows turns the counts into each row's
 //                 index u in a compact list of the step's rows.  A second pass
 //                 gathers the kept gradient rows of rows with two or more kept
-//                 occurrences (staged in shared memory with cp.async, all of a
-//                 round's rows in flight) and sums them with compensated
+//                 occurrences (staged in shared memory with cp.async, each lane
+//                 copying its own row, all of a round's rows in flight) and
+//                 sums them with compensated
 //                 (TwoSum) arithmetic, lane = element, in sorted order.  A row
 //                 with one kept occurrence needs no sum: its list entry points
 //                 at the message's gradient row.  Rows that cross a window
@@ -54,14 +55,15 @@ constexpr unsigned long long ST_INCL = 2ull << 30;
 constexpr unsigned long long ST_FLAGS = 3ull << 30;
 constexpr unsigned long long ST_COUNT = (1ull << 30) - 1;
 
-// Per warp: 32 staged gradient rows, then the window's row pointers and keys.
+// Per warp: one buffer of 32 staged gradient rows, then the window's keys and
+// occurrence indices (written by the first pass, read by the second).
 template <int EPL>
 struct ReduceCfg {
   static constexpr int WARPS = EPL <= 2 ? 8 : (EPL == 4 ? 4 : 2);
   static constexpr int THREADS = WARPS * 32;
-  static constexpr int MIN_BLOCKS = EPL <= 2 ? 3 : 2;
+  static constexpr int MIN_BLOCKS = EPL == 1 ? 4 : (EPL == 2 ? 3 : 2);
   static constexpr size_t WARP_BYTES =
-      (size_t)32 * 32 * EPL * sizeof(float) + (size_t)32 * WIN_ROUNDS * (8 + 4);
+      (size_t)32 * 32 * EPL * sizeof(float) + (size_t)32 * WIN_ROUNDS * 2 * sizeof(uint32_t);
   static constexpr size_t SMEM = (size_t)WARPS * WARP_BYTES;
 };
 __device__ __forceinline__ uint32_t ld_volatile_u32(const uint32_t* p) {
@@ -179,10 +181,10 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
   __shared__ uint32_t s_off[MSG_CACHE + 1];
   __shared__ int64_t s_tok[MSG_CACHE];
   __shared__ const float* s_rowp[MSG_CACHE];
-  __shared__ uint64_t s_bar[Cfg::WARPS];
   extern __shared__ __align__(128) unsigned char s_dyn[];
 
-  if (ld_volatile_u32(err.step) & (ERR_ID_RANGE | ERR_TIMEOUT)) return;
+  // block-uniform: another kernel may set the word while this block reads it
+  if (__syncthreads_or((ld_volatile_u32(err.step) & (ERR_ID_RANGE | ERR_TIMEOUT)) != 0u)) return;
   const int M = a.M;
   const uint32_t* off_g = a.msg_off + (size_t)tb.t * (M + 1);
   const float* const* rows_g = a.rows_ptr + (size_t)tb.t * M;
@@ -194,21 +196,15 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       s_rowp[i] = rows_g[i];
     }
   }
-  if (threadIdx.x < Cfg::WARPS) mbar_init(&s_bar[threadIdx.x], 1u);
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   __syncthreads();
   const uint32_t* off = cached ? s_off : off_g;
 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   constexpr int SS = 32 * EPL;  // staged row stride (floats)
   float* stage = reinterpret_cast<float*>(s_dyn + (size_t)warp * Cfg::WARP_BYTES);
-  const float** prow = reinterpret_cast<const float**>(stage + 32 * SS);  // per position
-  uint32_t* pkey = reinterpret_cast<uint32_t*>(prow + 32 * WIN_ROUNDS);
-  uint64_t* bar = &s_bar[warp];
-  uint32_t parity = 0u;
+  uint2* pkv = reinterpret_cast<uint2*>(stage + 32 * SS);  // [position in window]: key, occurrence
   const int d = tb.d;
-  const bool bulk = (d & 3) == 0;  // rows are 16-byte aligned: one bulk copy per row
-  const uint32_t row_bytes = (uint32_t)d * 4u;
+  const bool vec16 = (d & 3) == 0;  // gradient rows are 16-byte aligned
   const int64_t nbase = a.nbase[tb.t];
   const uint32_t n_t = (uint32_t)(tb.pos_end - tb.pos_begin);
   const uint32_t v_t = (uint32_t)tb.rows;
@@ -217,12 +213,23 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
 
   uint32_t n_pairs = 0, n_pairs_dropped = 0, n_kept_occ = 0, n_heads = 0;
   unsigned long long stale_sum = 0, stale_max = 0;
+  __shared__ uint32_t s_tile, s_base, s_cnt[Cfg::WARPS];
+  const int64_t n_tiles = (n_win + Cfg::WARPS - 1) / Cfg::WARPS;
 
+  // A block claims a tile of WARPS consecutive windows (in order, by ticket);
+  // warp j takes window WARPS * tile + j.
   for (;;) {
-    uint32_t w32 = 0;
-    if (lane == 0) w32 = atomicAdd(so.ticket, 1u);
-    const int64_t w = (int64_t)__shfl_sync(FULL, w32, 0);
-    if (w >= n_win) break;
+    if (threadIdx.x == 0) s_tile = atomicAdd(so.ticket, 1u);
+    __syncthreads();
+    const int64_t bt = (int64_t)s_tile;
+    if (bt >= n_tiles) break;
+    const int64_t w = bt * Cfg::WARPS + warp;
+    if (w >= n_win) {  // past the last window: only the barriers
+      s_cnt[warp] = 0u;
+      __syncthreads();
+      __syncthreads();
+      continue;
+    }
     const int64_t p0 = tb.pos_begin + w * wp;
     const int64_t p1 = (p0 + wp < tb.pos_end) ? p0 + wp : tb.pos_end;
     const int R = (int)((p1 - p0 + 31) >> 5);
@@ -239,6 +246,9 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
         vv[r] = vals[pos];
       }
     }
+#pragma unroll
+    for (int r = 0; r < WIN_ROUNDS; ++r)
+      if (r < R) pkv[32 * r + lane] = make_uint2(kk[r], vv[r]);
     // the neighbours outside the window: lane 0 the position before, lane 1 after
     uint32_t edge_k = NO_KEY, edge_v = 0u;
     if (lane == 0 && p0 > tb.pos_begin) {
@@ -266,10 +276,10 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       }
     }
     const bool cont_end = p1 < tb.pos_end && next_key == last_key;  // last row goes on
-    if (lane == 0)
-      st_relaxed_u64(so.status + w, ep | (w == 0 ? ST_INCL : ST_AGG) | (unsigned long long)nh);
+    const uint32_t key0 = __shfl_sync(FULL, kk[0], 0);
+    if (lane == 0) s_cnt[warp] = nh;
 
-    // ---- pass 1b: messages, tags, weights (Eq. (1)), flags, row pointers --------
+    // ---- pass 1b: messages, tags, weights (Eq. (1)), new-message flags ----------
     uint32_t mm[WIN_ROUNDS];
     int32_t tg[WIN_ROUNDS];
 #pragma unroll
@@ -302,17 +312,14 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
         const bool valid = mm[r] != 0xFFFFFFFEu;
         bool keep = false;
         uint32_t stale = 0u;
-        const float* rowp = nullptr;
         if (valid) {
           const uint32_t m = mm[r];
-          const uint32_t o_t = (uint32_t)((int64_t)vv[r] - nbase);
           const int64_t tok = cached ? s_tok[m] : a.tokens[m];
           const int64_t ref = a.row_staleness == 0 ? (int64_t)tg[r] : a.k;
           const int64_t diff = ref - tok;
           const uint64_t sl = diff > 0 ? (uint64_t)diff : 0ull;
           keep = sl <= (uint64_t)(int64_t)a.iota;
           stale = (uint32_t)(sl > 0xFFFFFFFFull ? 0xFFFFFFFFull : sl);
-          rowp = (cached ? s_rowp[m] : rows_g[m]) + (size_t)(o_t - off[m]) * (size_t)d;
         }
         uint32_t pm = __shfl_up_sync(FULL, mm[r], 1);
         if (lane == 0) pm = prev_m;
@@ -331,48 +338,64 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
           myK = Km;
           myN = Nm;
         }
-        prow[32 * r + lane] = rowp;
-        pkey[32 * r + lane] = kk[r];
         prev_m = __shfl_sync(FULL, mm[r], 31);
       }
     }
 
-    // ---- look back for the window's first list index -----------------------------
-    uint32_t prefix = 0u;
-    if (w > 0) {
-      int64_t j = w - 1;
-      const uint64_t t0 = globaltimer_ns();
-      for (;;) {
-        const int64_t q = j - lane;
-        unsigned long long v = ep | ST_INCL;  // before window 0: nothing
-        if (q >= 0) v = ld_relaxed_u64(so.status + q);
-        const bool ready = (v & ~0xFFFFFFFFull) == ep && (v & ST_FLAGS) != 0ull;
-        const bool incl = ready && (v & ST_INCL) != 0ull;
-        const uint32_t rm = __ballot_sync(FULL, ready), im = __ballot_sync(FULL, incl);
-        const int first_nr = ~rm ? __ffs(~rm) - 1 : 32;
-        const int first_in = im ? __ffs(im) - 1 : 32;
-        const int take = first_in < first_nr ? first_in + 1 : first_nr;
-        uint32_t c = lane < take ? (uint32_t)(v & ST_COUNT) : 0u;
+    // ---- the window's first list index: warp 0 looks back over block tiles
+    __syncthreads();
+    if (warp == 0) {
+      uint32_t c = lane < Cfg::WARPS ? s_cnt[lane] : 0u;
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(FULL, c, o);
-        prefix += c;
-        if (first_in < first_nr) break;
-        j -= take;
-        if (take == 0 && ((ld_volatile_u32(err.step) & ERR_TIMEOUT) ||
-                          (int64_t)(globaltimer_ns() - t0) > wait_ns)) {
-          if (lane == 0) raise_error(err, ERR_TIMEOUT);
-          break;
-        }
-      }
+      for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(FULL, c, o);
+      const uint32_t tile_cnt = c;
       if (lane == 0)
-        st_relaxed_u64(so.status + w,
-                       ep | ST_INCL | (unsigned long long)((prefix + nh) & ST_COUNT));
+        st_relaxed_u64(so.status + bt,
+                       ep | (bt == 0 ? ST_INCL : ST_AGG) | (unsigned long long)tile_cnt);
+      uint32_t tp = 0u;
+      if (bt > 0) {
+        int64_t j = bt - 1;
+        const uint64_t t0 = globaltimer_ns();
+        for (;;) {
+          const int64_t q = j - lane;
+          unsigned long long v = ep | ST_INCL;  // before tile 0: nothing
+          if (q >= 0) v = ld_relaxed_u64(so.status + q);
+          const bool ready = (v & ~0xFFFFFFFFull) == ep && (v & ST_FLAGS) != 0ull;
+          const bool incl = ready && (v & ST_INCL) != 0ull;
+          const uint32_t rm = __ballot_sync(FULL, ready), im = __ballot_sync(FULL, incl);
+          const int first_nr = ~rm ? __ffs(~rm) - 1 : 32;
+          const int first_in = im ? __ffs(im) - 1 : 32;
+          const int take = first_in < first_nr ? first_in + 1 : first_nr;
+          uint32_t cc = lane < take ? (uint32_t)(v & ST_COUNT) : 0u;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) cc += __shfl_xor_sync(FULL, cc, o);
+          tp += cc;
+          if (first_in < first_nr) break;
+          j -= take;
+          if (take == 0 && ((ld_volatile_u32(err.step) & ERR_TIMEOUT) ||
+                            (int64_t)(globaltimer_ns() - t0) > wait_ns)) {
+            if (lane == 0) raise_error(err, ERR_TIMEOUT);
+            break;
+          }
+        }
+        if (lane == 0)
+          st_relaxed_u64(so.status + bt,
+                         ep | ST_INCL | (unsigned long long)((tp + tile_cnt) & ST_COUNT));
+      }
+      if (lane == 0) {
+        s_base = tp;
+        if (bt == n_tiles - 1) *so.total = tp + tile_cnt;
+      }
     }
-    if (w == n_win - 1 && lane == 0) *so.total = prefix + nh;
+    __syncthreads();
+    uint32_t prefix = s_base;
+    for (int j = 0; j < warp; ++j) prefix += s_cnt[j];
     n_heads += nh;
-    __syncwarp();
 
     // ---- pass 2: gather and sum, round by round ----------------------------------
+    // prepare() analyses a round, writes the list entries of rows that begin
+    // and end inside it and issues its gathers; the sums follow in order and
+    // carry the open row from round to round.
     CSum acc[EPL];
 #pragma unroll
     for (int e = 0; e < EPL; ++e) acc[e] = CSum{0.f, 0.f};
@@ -380,10 +403,17 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
     uint32_t ox = 0u, ou = 0u, ohead = 0u;
     bool open_head = false;  // the open row's head lies in this window
     bool wrote_slot0 = false;
-    uint32_t hb = 0u;  // heads of the window before this round
+    uint32_t hb = 0u;  // heads of the window before the next round to prepare
     if (p0 > tb.pos_begin && !(__shfl_sync(FULL, myH, 0) & 1u))
-      ox = pkey[0] - tb.key_base;  // a row that began in an earlier window is open
-    for (int r = 0; r < R; ++r) {
+      ox = key0 - tb.key_base;  // a row that began in an earlier window is open
+
+    struct Round {
+      uint32_t Hm, Km, Nm, Gm, Fm, u_fl, key, hb;
+      int n_round;
+      bool cont;
+    };
+    auto prepare = [&](int r, float* buf) -> Round {
+      Round st;
       const int64_t rb = p0 + 32 * r;
       const int n_round = (int)((p1 - rb) < 32 ? (p1 - rb) : 32);
       const uint32_t Hm = __shfl_sync(FULL, myH, r);
@@ -393,8 +423,18 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       const uint32_t Hn = __shfl_sync(FULL, myH, r + 1 < 32 ? r + 1 : 31);
       const bool cont = (r + 1 < R) ? !(Hn & 1u) : cont_end;  // the round's last row goes on
       const bool valid = lane < n_round;
-      const uint32_t key = valid ? pkey[32 * r + lane] : NO_KEY;
-      const float* rowp = valid ? prow[32 * r + lane] : nullptr;
+      // lane metadata again, from the keys and occurrences pass 1 kept
+      uint32_t key = NO_KEY;
+      const float* rowp = nullptr;
+      if (valid) {
+        const uint2 kv = pkv[32 * r + lane];
+        key = kv.x;
+        const uint32_t o_t = (uint32_t)((int64_t)kv.y - nbase);
+        if (o_t < n_t) {
+          const uint32_t m = (uint32_t)message_of_any(off, M, o_t);
+          rowp = (cached ? s_rowp[m] : rows_g[m]) + (size_t)(o_t - off[m]) * (size_t)d;
+        }
+      }
       const bool keep = (Km >> lane) & 1u;
       // pieces: maximal runs of one row inside the round
       const uint32_t Bm = (Hm | 1u) & Vm;
@@ -410,7 +450,7 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       const uint32_t ca = __popc(Nm & rng), ck = __popc(Nm & Km & rng);
       // rows that begin and end inside the round: the lane of the head writes
       // the list entry -- pointing at the single kept gradient row, or at the
-      // compact slot that the sum below fills
+      // compact slot that the sum fills
       const bool single = starts && is_head && closes && kc <= 1u;
       const bool local_sum = starts && is_head && closes && kc >= 2u;
       const uint32_t u_me = prefix + hb + __popc(Hm & lanemask_lt());
@@ -431,38 +471,63 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       // kept position of a local sum, which also learns the row's list index
       const bool gather = valid && keep && !((Sm >> s_of) & 1u);
       const bool flush = gather && ((Lm >> s_of) & 1u) && (31 - __clz(kmask)) == lane;
-      const uint32_t Gm = __ballot_sync(FULL, gather);
-      const uint32_t Fm = __ballot_sync(FULL, flush);
-      const uint32_t u_fl = __shfl_sync(FULL, u_me, s_of);
-      if (Gm) {
-        if (bulk) {
-          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-          if (lane == 0) mbar_arrive_expect_tx(bar, (uint32_t)__popc(Gm) * row_bytes);
-          __syncwarp();
-          if (gather) bulk_g2s(stage + lane * SS, rowp, row_bytes, bar);
-          if (!mbar_wait(bar, parity, wait_ns)) {
-            if (lane == 0) raise_error(err, ERR_TIMEOUT);
-            mbar_wait(bar, parity, 1000000000ll);  // let issued copies land (bounded)
-          }
-          parity ^= 1u;
+      st.Gm = __ballot_sync(FULL, gather);
+      st.Fm = __ballot_sync(FULL, flush);
+      st.u_fl = __shfl_sync(FULL, u_me, s_of);
+      if (gather) {  // each gathering lane copies its own row
+        float* dst = buf + lane * SS;
+        if (vec16) {
+          for (int q = 0; q < d; q += 4)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst + q)),
+                         "l"(rowp + q)
+                         : "memory");
         } else {
-          uint32_t gm = Gm;
-          while (gm) {
-            const int j = __ffs(gm) - 1;
-            gm &= gm - 1u;
-            const float* src = (const float*)__shfl_sync(FULL, (unsigned long long)rowp, j);
-            for (int q = lane; q < d; q += 32)
-              asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
-                               smem_addr(stage + j * SS + q)),
-                           "l"(src + q)
-                           : "memory");
-          }
-          asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+          for (int q = 0; q < d; ++q)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(dst + q)),
+                         "l"(rowp + q)
+                         : "memory");
         }
       }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      st.Hm = Hm;
+      st.Km = Km;
+      st.Nm = Nm;
+      st.key = __shfl_sync(FULL, key, 31 - __clz(Bm));  // key where the round's last piece starts
+      st.hb = hb;
+      st.n_round = n_round;
+      st.cont = cont;
+      hb += __popc(Hm);
+      return st;
+    };
+
+    for (int r = 0; r < R; ++r) {
+      float* buf = stage;
+      const Round cur = prepare(r, buf);
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
       __syncwarp();
+      const uint32_t Hm = cur.Hm, Km = cur.Km, Nm = cur.Nm, Gm = cur.Gm, Fm = cur.Fm;
+      const int n_round = cur.n_round;
+      const bool cont = cur.cont;
+      const uint32_t Vm = bits_below(n_round);
+      const uint32_t Bm = (Hm | 1u) & Vm;
+      const int64_t rb = p0 + 32 * r;
       // ---- the sums, lane = element, in sorted order
       uint32_t gm = Gm;
+      if (Hm == 0u) {
+        // The whole round continues the open row (a Zipf-hot row): the same
+        // compensated sum in the same order, unrolled, positions that were not
+        // gathered adding an exact zero.
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const bool on = (Gm >> j) & 1u;
+#pragma unroll
+          for (int q = 0; q < EPL; ++q) {
+            const float x = buf[j * SS + lane * EPL + q];
+            csum_add(acc[q], on ? x : 0.f);
+          }
+        }
+        gm = 0u;
+      }
       if (!(Hm & 1u)) {  // position 0 continues the open row
         const uint32_t a0 = Bm & ~1u;
         const int e0 = a0 ? __ffs(a0) - 1 : n_round;
@@ -472,7 +537,7 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
         while (g0) {
           const int j = __ffs(g0) - 1;
           g0 &= g0 - 1u;
-          const float* sp = stage + j * SS + lane * EPL;
+          const float* sp = buf + j * SS + lane * EPL;
 #pragma unroll
           for (int q = 0; q < EPL; ++q) csum_add(acc[q], sp[q]);
         }
@@ -486,6 +551,8 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
           } else {
             write_record<EPL>(so, w, 0, d, REC_CLOSED, ox, rc, 0u, 0u, lane, acc);
             wrote_slot0 = true;
+            // the row's head is the last one before this window: list index prefix - 1
+            if (lane == 0 && prefix > 0u) so.cross_end[prefix - 1u] = (uint32_t)w;
           }
           open_head = false;
 #pragma unroll
@@ -495,11 +562,11 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       while (gm) {
         const int j = __ffs(gm) - 1;
         gm &= gm - 1u;
-        const float* sp = stage + j * SS + lane * EPL;
+        const float* sp = buf + j * SS + lane * EPL;
 #pragma unroll
         for (int q = 0; q < EPL; ++q) csum_add(acc[q], sp[q]);
         if ((Fm >> j) & 1u) {
-          const uint32_t uj = __shfl_sync(FULL, u_fl, j);
+          const uint32_t uj = __shfl_sync(FULL, cur.u_fl, j);
           float* dst = so.compact + (size_t)uj * so.cs;
 #pragma unroll
           for (int q = 0; q < EPL; ++q) {
@@ -513,15 +580,14 @@ __global__ void __launch_bounds__(ReduceCfg<EPL>::THREADS, ReduceCfg<EPL>::MIN_B
       const int ls = 31 - __clz(Bm);
       if (cont && ((Hm >> ls) & 1u)) {
         const uint32_t rl = Vm & bits_from(ls);
-        ox = __shfl_sync(FULL, key, ls) - tb.key_base;
-        ou = prefix + hb + __popc(Hm & bits_below(ls));
+        ox = cur.key - tb.key_base;
+        ou = prefix + cur.hb + __popc(Hm & bits_below(ls));
         ohead = (uint32_t)(rb + ls);
         rc = RunCounts{(uint32_t)__popc(Nm & rl), (uint32_t)__popc(Nm & Km & rl),
                        (uint32_t)__popc(Km & rl)};
         open_head = true;
       }
-      hb += __popc(Hm);
-      __syncwarp();
+      __syncwarp();  // the buffer is refilled by the next round
     }
     bool wrote_slot1 = false;
     if (cont_end) {  // the open row goes on in the next window
@@ -572,60 +638,28 @@ __device__ __forceinline__ void cross_row(const StepArgs& a, const SegTable& tb,
                                           uint32_t* dbg_kept, const ErrSink& err) {
   __shared__ float s_hi[CROSS_WARPS][32 * EPL];
   __shared__ float s_lo[CROSS_WARPS][32 * EPL];
-  __shared__ int s_first;
   __shared__ uint32_t s_bad, s_call, s_ckept, s_kocc;
   const uint32_t* m1 = so.rec_meta + ((size_t)w * 2 + 1) * REC_META;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (m1[0] != REC_OWNER) {  // cannot happen: the list holds owners only
-    if (tid == 0) raise_error(err, ERR_INTERNAL);
-    return;
-  }
-  const uint32_t x = m1[1], head_pos = m1[5], u = m1[6];
+  const uint32_t type = m1[0], x = m1[1], head_pos = m1[5], u = m1[6];
+  const int64_t end = type == REC_OWNER ? (int64_t)so.cross_end[u] : -1;
   if (tid == 0) {
     s_bad = 0u;
     s_call = m1[2];
     s_ckept = m1[3];
     s_kocc = m1[4];
   }
-  // Find the window where the row ends: every record before it must carry the
-  // row on (PASS), the last one closes it (CLOSED).
-  int64_t end = -1;
-  for (int64_t base = w + 1; base < n_win; base += CROSS_THREADS) {
-    if (tid == 0) s_first = CROSS_THREADS;
-    __syncthreads();
-    const int64_t q = base + tid;
-    uint32_t ty = REC_NONE, rx = 0u;
-    const uint32_t* m0 = nullptr;
-    if (q < n_win) {
-      m0 = so.rec_meta + ((size_t)q * 2 + 0) * REC_META;
-      ty = m0[0];
-      rx = m0[1];
-    }
-    if (q < n_win && ty == REC_CLOSED && rx == x) atomicMin(&s_first, tid);
-    __syncthreads();
-    const int first = s_first;
-    if (tid < first && (q >= n_win || ty != REC_PASS || rx != x)) s_bad = 1u;
-    if (tid <= first && q < n_win && rx == x && (ty == REC_PASS || ty == REC_CLOSED)) {
-      atomicAdd(&s_call, m0[2]);
-      atomicAdd(&s_ckept, m0[3]);
-      atomicAdd(&s_kocc, m0[4]);
-    }
-    __syncthreads();
-    if (first < CROSS_THREADS) {
-      end = base + first;
-      break;
-    }
-    if (s_bad) break;
-  }
   __syncthreads();
-  if (end < 0 || s_bad || x >= (uint32_t)tb.rows) {
+  // the list holds owners only; the row ends in a later window
+  if (end <= w || end >= n_win || x >= (uint32_t)tb.rows) {
     if (tid == 0) raise_error(err, ERR_INTERNAL);
     __syncthreads();
     return;
   }
   // Merge the partial sums: warp j takes the records of windows w+1+j,
-  // w+1+j+8, ... in order (warp 0 starts from the owner's), then warp 0 merges
-  // the warps' results in warp order.
+  // w+1+j+W, ... in order (warp 0 starts from the owner's), then warp 0 merges
+  // the warps' results in warp order.  Each record must carry the row on
+  // (PASS) but the last, which closes it (CLOSED).
   const int d = tb.d;
   const int64_t R = end - w;
   CSum acc[EPL];
@@ -639,13 +673,16 @@ __device__ __forceinline__ void cross_row(const StepArgs& a, const SegTable& tb,
       if (el < d) acc[e] = CSum{so.rec_hi[b + el], so.rec_lo[b + el]};
     }
   }
-  constexpr int U4 = EPL <= 2 ? 8 : 4;  // records in flight per warp
+  constexpr int U4 = EPL == 1 ? 8 : (EPL == 2 ? 4 : 2);  // records in flight per warp
+  uint32_t c_all = 0u, c_kept = 0u, k_occ = 0u;
+  bool bad = false;
   for (int64_t i0 = warp; i0 < R; i0 += CROSS_WARPS * U4) {
     float hi[U4][EPL], lo[U4][EPL];
 #pragma unroll
     for (int k = 0; k < U4; ++k) {
       const int64_t i = i0 + (int64_t)k * CROSS_WARPS;
-      const size_t b = ((size_t)(w + 1 + i) * 2 + 0) * (size_t)so.rec_stride;
+      const size_t rw = (size_t)(w + 1 + i) * 2 + 0;
+      const size_t b = rw * (size_t)so.rec_stride;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) {
         const int el = lane * EPL + e;
@@ -656,6 +693,14 @@ __device__ __forceinline__ void cross_row(const StepArgs& a, const SegTable& tb,
           lo[k][e] = so.rec_lo[b + el];
         }
       }
+      if (i < R && lane == 0) {
+        const uint32_t* m0 = so.rec_meta + rw * REC_META;
+        const uint32_t want = i + 1 == R ? REC_CLOSED : REC_PASS;
+        if (m0[0] != want || m0[1] != x) bad = true;
+        c_all += m0[2];
+        c_kept += m0[3];
+        k_occ += m0[4];
+      }
     }
 #pragma unroll
     for (int k = 0; k < U4; ++k)
@@ -664,6 +709,12 @@ __device__ __forceinline__ void cross_row(const StepArgs& a, const SegTable& tb,
         for (int e = 0; e < EPL; ++e) csum_merge(acc[e], hi[k][e], lo[k][e]);
       }
   }
+  if (lane == 0) {
+    if (bad) s_bad = 1u;
+    atomicAdd(&s_call, c_all);
+    atomicAdd(&s_ckept, c_kept);
+    atomicAdd(&s_kocc, k_occ);
+  }
 #pragma unroll
   for (int e = 0; e < EPL; ++e) {
     s_hi[warp][lane * EPL + e] = acc[e].hi;
@@ -671,14 +722,18 @@ __device__ __forceinline__ void cross_row(const StepArgs& a, const SegTable& tb,
   }
   __syncthreads();
   if (warp == 0) {
+    if (s_bad) {
+      if (lane == 0) raise_error(err, ERR_INTERNAL);
+    } else {
 #pragma unroll
-    for (int j = 1; j < CROSS_WARPS; ++j)
+      for (int j = 1; j < CROSS_WARPS; ++j)
 #pragma unroll
-      for (int e = 0; e < EPL; ++e)
-        csum_merge(acc[e], s_hi[j][lane * EPL + e], s_lo[j][lane * EPL + e]);
-    const RunCounts rc{s_call, s_ckept, s_kocc};
-    finish_local_row<EPL>(so, d, a.sparse_den, a.M, x, u, head_pos, rc, acc, lane, dbg_count,
-                          dbg_kept);
+        for (int e = 0; e < EPL; ++e)
+          csum_merge(acc[e], s_hi[j][lane * EPL + e], s_lo[j][lane * EPL + e]);
+      const RunCounts rc{s_call, s_ckept, s_kocc};
+      finish_local_row<EPL>(so, d, a.sparse_den, a.M, x, u, head_pos, rc, acc, lane, dbg_count,
+                            dbg_kept);
+    }
   }
   __syncthreads();  // the shared scratch is reused by the block's next row
 }
@@ -686,10 +741,10 @@ __device__ __forceinline__ void cross_row(const StepArgs& a, const SegTable& tb,
 // One block per listed row (the list order does not matter: rows are
 // independent and each row's merge order is fixed).
 template <int EPL>
-__global__ void __launch_bounds__(CROSS_THREADS)
+__global__ void __launch_bounds__(CROSS_THREADS, EPL <= 2 ? 4 : 2)
     k_seg_cross(StepArgs a, SegTable tb, SegOut so, int64_t n_win, uint32_t* dbg_count,
                 uint32_t* dbg_kept, ErrSink err) {
-  if (ld_volatile_u32(err.step)) return;
+  if (__syncthreads_or(ld_volatile_u32(err.step) != 0u)) return;
   const uint32_t n = ld_volatile_u32(so.cross_count);
   for (uint32_t i = blockIdx.x; i < n; i += gridDim.x)
     cross_row<EPL>(a, tb, so, n_win, (int64_t)so.cross_list[i], dbg_count, dbg_kept, err);
@@ -700,12 +755,110 @@ __global__ void __launch_bounds__(CROSS_THREADS)
 // ---------------------------------------------------------------------------
 constexpr int UPD_THREADS = 256;
 
+// One row's pieces held by a lane: gradient, weights, optimizer state.
+template <int NV>
+struct RowRegs {
+  float g[NV], w[NV], s0[NV], s1[NV];
+};
+
+struct RowRef {
+  const float* src;
+  uint32_t x;
+  float den;
+  bool act;
+};
+
+__device__ __forceinline__ RowRef load_ref(const SegOut& so, int64_t u, uint32_t U) {
+  RowRef r{nullptr, 0u, 0.f, false};
+  if (u < (int64_t)U) {
+    const ulonglong2 v = *reinterpret_cast<const ulonglong2*>(so.desc + u);
+    r.src = (const float*)v.x;
+    r.x = (uint32_t)v.y;
+    r.den = __uint_as_float((uint32_t)(v.y >> 32));
+    r.act = r.den > 0.f;
+  }
+  return r;
+}
+
+template <int CH, int CPL>
+__device__ __forceinline__ void load_row(const SegTable& tb, const RowRef& r, int l, int L, int C,
+                                         bool adam, RowRegs<CH * CPL>& v) {
+  if (!r.act) return;
+  const int d = tb.d;
+#pragma unroll
+  for (int c = 0; c < CPL; ++c) {
+    const int q = l + c * L;
+    if (q < C) {
+      const size_t o = (size_t)r.x * d + (size_t)q * CH;
+      if constexpr (CH == 4) {
+        const float4 g4 = *reinterpret_cast<const float4*>(r.src + q * 4);
+        const float4 w4 = *reinterpret_cast<const float4*>(tb.w + o);
+        const float4 a4 = *reinterpret_cast<const float4*>(tb.s0 + o);
+        v.g[4 * c] = g4.x; v.g[4 * c + 1] = g4.y; v.g[4 * c + 2] = g4.z; v.g[4 * c + 3] = g4.w;
+        v.w[4 * c] = w4.x; v.w[4 * c + 1] = w4.y; v.w[4 * c + 2] = w4.z; v.w[4 * c + 3] = w4.w;
+        v.s0[4 * c] = a4.x; v.s0[4 * c + 1] = a4.y; v.s0[4 * c + 2] = a4.z; v.s0[4 * c + 3] = a4.w;
+        if (adam) {
+          const float4 b4 = *reinterpret_cast<const float4*>(tb.s1 + o);
+          v.s1[4 * c] = b4.x; v.s1[4 * c + 1] = b4.y; v.s1[4 * c + 2] = b4.z; v.s1[4 * c + 3] = b4.w;
+        }
+      } else {
+        v.g[c] = r.src[q];
+        v.w[c] = tb.w[o];
+        v.s0[c] = tb.s0[o];
+        if (adam) v.s1[c] = tb.s1[o];
+      }
+    }
+  }
+}
+
+template <int CH, int CPL>
+__device__ __forceinline__ void update_row(const SegTable& tb, const RowRef& r, int l, int L, int C,
+                                           bool adam, int32_t tag, RowRegs<CH * CPL>& v,
+                                           uint32_t& applied) {
+  if (!r.act) return;
+  const int d = tb.d;
+#pragma unroll
+  for (int c = 0; c < CPL; ++c) {
+    const int q = l + c * L;
+    if (q >= C) continue;
+#pragma unroll
+    for (int k = 0; k < CH; ++k) {
+      const int i = c * CH + k;
+      float b = adam ? v.s1[i] : 0.f;
+      const float gi = r.den == 1.0f ? v.g[i] : __fdiv_rn(v.g[i], r.den);
+      opt_update(tb.opt, v.w[i], v.s0[i], b, gi);
+      v.s1[i] = b;
+    }
+    const size_t o = (size_t)r.x * d + (size_t)q * CH;
+    if constexpr (CH == 4) {
+      const int i = 4 * c;
+      *reinterpret_cast<float4*>(tb.w + o) = make_float4(v.w[i], v.w[i + 1], v.w[i + 2], v.w[i + 3]);
+      *reinterpret_cast<float4*>(tb.s0 + o) =
+          make_float4(v.s0[i], v.s0[i + 1], v.s0[i + 2], v.s0[i + 3]);
+      if (adam)
+        *reinterpret_cast<float4*>(tb.s1 + o) =
+            make_float4(v.s1[i], v.s1[i + 1], v.s1[i + 2], v.s1[i + 3]);
+    } else {
+      tb.w[o] = v.w[c];
+      tb.s0[o] = v.s0[c];
+      if (adam) tb.s1[o] = v.s1[c];
+    }
+  }
+  if (l == 0) {
+    tb.ver[r.x] = tag;
+    ++applied;
+  }
+}
+
 // CH floats per piece (4: 16-byte pieces, rows with d % 4 == 0; else 1), at
-// most CPL pieces per lane.
+// most CPL pieces per lane.  Each lane group walks its rows with the next
+// row's loads issued before the current row's update (and the list entry two
+// rows ahead), so memory latency overlaps the optimizer arithmetic.
 template <int CH, int CPL>
 __global__ void __launch_bounds__(UPD_THREADS, (CH == 4 && CPL == 1) || (CH == 1 && CPL <= 2) ? 4 : 2)
     k_row_update(StepArgs a, SegTable tb, SegOut so, DevStats* st, ErrSink err) {
-  if (ld_volatile_u32(err.step)) return;  // a failed step changes no row
+  // a failed step changes no row (warp-uniform: the warp reduces at the end)
+  if (__any_sync(FULL, ld_volatile_u32(err.step) != 0u)) return;
   const uint32_t U = ld_volatile_u32(so.total);
   const int d = tb.d;
   const int C = d / CH;  // pieces per row
@@ -719,86 +872,18 @@ __global__ void __launch_bounds__(UPD_THREADS, (CH == 4 && CPL == 1) || (CH == 1
   const int64_t TG = (int64_t)gridDim.x * (UPD_THREADS / 32) * G;
   const bool adam = tb.opt.kind == 1;
   const int32_t tag = (int32_t)(a.k + 1);
-  constexpr int NV = CH * CPL;
   uint32_t applied = 0u;
-  const ulonglong2 zero = make_ulonglong2(0ull, 0ull);
-  int64_t ua = gw * G + g;
-  // descriptors of the next iteration are loaded one iteration ahead
-  ulonglong2 na = ua < (int64_t)U ? *reinterpret_cast<const ulonglong2*>(so.desc + ua) : zero;
-  ulonglong2 nb = ua + TG < (int64_t)U ? *reinterpret_cast<const ulonglong2*>(so.desc + ua + TG) : zero;
-  for (; ua < (int64_t)U; ua += 2 * TG) {
-    const int64_t ub = ua + TG;
-    const ulonglong2 da = na, db = nb;
-    {
-      const int64_t uc = ua + 2 * TG;
-      na = uc < (int64_t)U ? *reinterpret_cast<const ulonglong2*>(so.desc + uc) : zero;
-      nb = uc + TG < (int64_t)U ? *reinterpret_cast<const ulonglong2*>(so.desc + uc + TG) : zero;
-    }
-    const float* src[2] = {(const float*)da.x, (const float*)db.x};
-    const uint32_t xr[2] = {(uint32_t)da.y, (uint32_t)db.y};
-    const float den[2] = {__uint_as_float((uint32_t)(da.y >> 32)),
-                          __uint_as_float((uint32_t)(db.y >> 32))};
-    const bool act[2] = {den[0] > 0.f, ub < (int64_t)U && den[1] > 0.f};
-    float gv[2][NV], wv[2][NV], av[2][NV], bv[2][NV];
-#pragma unroll
-    for (int h = 0; h < 2; ++h)
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) {
-        const int q = l + c * L;
-        if (act[h] && q < C) {
-          const size_t r = (size_t)xr[h] * d + (size_t)q * CH;
-          if constexpr (CH == 4) {
-            const float4 g4 = *reinterpret_cast<const float4*>(src[h] + q * 4);
-            const float4 w4 = *reinterpret_cast<const float4*>(tb.w + r);
-            const float4 a4 = *reinterpret_cast<const float4*>(tb.s0 + r);
-            gv[h][4 * c] = g4.x; gv[h][4 * c + 1] = g4.y; gv[h][4 * c + 2] = g4.z; gv[h][4 * c + 3] = g4.w;
-            wv[h][4 * c] = w4.x; wv[h][4 * c + 1] = w4.y; wv[h][4 * c + 2] = w4.z; wv[h][4 * c + 3] = w4.w;
-            av[h][4 * c] = a4.x; av[h][4 * c + 1] = a4.y; av[h][4 * c + 2] = a4.z; av[h][4 * c + 3] = a4.w;
-            if (adam) {
-              const float4 b4 = *reinterpret_cast<const float4*>(tb.s1 + r);
-              bv[h][4 * c] = b4.x; bv[h][4 * c + 1] = b4.y; bv[h][4 * c + 2] = b4.z; bv[h][4 * c + 3] = b4.w;
-            }
-          } else {
-            gv[h][c] = src[h][q];
-            wv[h][c] = tb.w[r];
-            av[h][c] = tb.s0[r];
-            if (adam) bv[h][c] = tb.s1[r];
-          }
-        }
-      }
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      if (!act[h]) continue;
-#pragma unroll
-      for (int c = 0; c < CPL; ++c) {
-        const int q = l + c * L;
-        if (q >= C) continue;
-#pragma unroll
-        for (int k = 0; k < CH; ++k) {
-          const int i = c * CH + k;
-          float b = adam ? bv[h][i] : 0.f;
-          const float gi = den[h] == 1.0f ? gv[h][i] : __fdiv_rn(gv[h][i], den[h]);
-          opt_update(tb.opt, wv[h][i], av[h][i], b, gi);
-          bv[h][i] = b;
-        }
-        const size_t r = (size_t)xr[h] * d + (size_t)q * CH;
-        if constexpr (CH == 4) {
-          const int i = 4 * c;
-          *reinterpret_cast<float4*>(tb.w + r) = make_float4(wv[h][i], wv[h][i + 1], wv[h][i + 2], wv[h][i + 3]);
-          *reinterpret_cast<float4*>(tb.s0 + r) = make_float4(av[h][i], av[h][i + 1], av[h][i + 2], av[h][i + 3]);
-          if (adam)
-            *reinterpret_cast<float4*>(tb.s1 + r) = make_float4(bv[h][i], bv[h][i + 1], bv[h][i + 2], bv[h][i + 3]);
-        } else {
-          tb.w[r] = wv[h][c];
-          tb.s0[r] = av[h][c];
-          if (adam) tb.s1[r] = bv[h][c];
-        }
-      }
-      if (l == 0) {
-        tb.ver[xr[h]] = tag;
-        ++applied;
-      }
-    }
+  int64_t u = gw * G + g;
+  RowRef cur = load_ref(so, u, U), nxt = load_ref(so, u + TG, U);
+  RowRegs<CH * CPL> vc, vn;
+  load_row<CH, CPL>(tb, cur, l, L, C, adam, vc);
+  for (; u < (int64_t)U; u += TG) {
+    const RowRef n2 = load_ref(so, u + 2 * TG, U);
+    load_row<CH, CPL>(tb, nxt, l, L, C, adam, vn);
+    update_row<CH, CPL>(tb, cur, l, L, C, adam, tag, vc, applied);
+    cur = nxt;
+    nxt = n2;
+    vc = vn;
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) applied += __shfl_xor_sync(FULL, applied, o);
@@ -810,8 +895,8 @@ __global__ void __launch_bounds__(UPD_THREADS, (CH == 4 && CPL == 1) || (CH == 1
 // ---------------------------------------------------------------------------
 template <typename K>
 int blocks_per_sm(K kernel, int threads, size_t smem) {
-  if (smem > 48 * 1024)
-    cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  // static + dynamic shared memory may pass 48 KB: always raise the limit
+  cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   int b = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, kernel, threads, smem) != cudaSuccess ||
       b < 1)
@@ -858,7 +943,7 @@ void launch_update_cfg(const StepArgs& a, const SegTable& tb, const SegOut& so, 
   const int C = tb.d / CH;
   int L = 1;
   while (L < C && L < 32) L <<= 1;
-  const int64_t rows_per_block = (int64_t)(UPD_THREADS / 32) * (32 / L) * 2;
+  const int64_t rows_per_block = (int64_t)(UPD_THREADS / 32) * (32 / L) * 2;  // two per group at least
   const int64_t grid =
       std::max<int64_t>(1, std::min<int64_t>((int64_t)num_sms * bps, (Nt + rows_per_block - 1) / rows_per_block));
   k_row_update<CH, CPL><<<(unsigned)grid, UPD_THREADS, 0, s>>>(a, tb, so, stats, err);
@@ -888,7 +973,7 @@ void launch_seg_cross(const StepArgs& a, const SegTable& tb, const SegOut& so, i
                       uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, cudaStream_t s) {
   if (n_win < 2) return;  // one window: no row can cross
   // at most one listed row per window but the last
-  const unsigned grid = (unsigned)std::min<int64_t>(n_win - 1, 2048);
+  const unsigned grid = (unsigned)std::min<int64_t>(n_win - 1, 152 * 8);
   const int d = tb.d;
   if (d <= 32)
     k_seg_cross<1><<<grid, CROSS_THREADS, 0, s>>>(a, tb, so, n_win, dbg_count, dbg_kept, err);

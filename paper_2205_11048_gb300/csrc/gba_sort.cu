@@ -21,8 +21,9 @@ namespace {
 constexpr int RADIX = 256;
 constexpr int SORT_THREADS = 256;  // one thread per digit in the look-back
 constexpr int SORT_WARPS = SORT_THREADS / 32;
-constexpr int SORT_ITEMS = 16;
-constexpr int SORT_TILE = SORT_THREADS * SORT_ITEMS;
+constexpr int SORT_ITEMS = SORT_TILE_KEYS / SORT_THREADS;
+constexpr int SORT_TILE = SORT_TILE_KEYS;
+static_assert(SORT_TILE_KEYS % SORT_THREADS == 0, "tile must fill the block");
 constexpr int MAX_PASSES = 4;
 constexpr int LB_WIN = 8;  // look-back window
 constexpr int OFF_CACHE = 1024;  // message offsets kept in shared memory
@@ -165,10 +166,12 @@ __global__ void __launch_bounds__(256) k_message_weights(StepArgs a, StepScratch
 }
 
 // ---------------------------------------------------------------------------
-// Digit counts of every pass in one read of the ids.
+// Digit counts of every pass in one read of the ids; also writes every
+// occurrence's key (keys0) for the first onesweep pass.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(SORT_THREADS) k_sort_histogram(StepArgs a, int passes,
-                                                                 StepScratch sc, ErrSink err) {
+                                                                 StepScratch sc, uint32_t* keys0,
+                                                                 ErrSink err) {
   __shared__ uint32_t h[MAX_PASSES][RADIX];
   __shared__ uint32_t s_off[OFF_CACHE];
   for (int i = threadIdx.x; i < MAX_PASSES * RADIX; i += SORT_THREADS) (&h[0][0])[i] = 0u;
@@ -177,6 +180,7 @@ __global__ void __launch_bounds__(SORT_THREADS) k_sort_histogram(StepArgs a, int
   const int64_t stride = (int64_t)gridDim.x * SORT_THREADS;
   for (int64_t o = (int64_t)blockIdx.x * SORT_THREADS + threadIdx.x; o < a.N; o += stride) {
     const uint32_t key = occurrence_key(a, offs, o, err);
+    keys0[o] = key;
     for (int p = 0; p < passes; ++p) atomicAdd(&h[p][(key >> (8 * p)) & (RADIX - 1)], 1u);
   }
   __syncthreads();
@@ -202,18 +206,16 @@ __global__ void __launch_bounds__(SORT_THREADS)
   __shared__ uint32_t s_keys[SORT_TILE];
   __shared__ uint32_t s_vals[SORT_TILE];
   __shared__ uint32_t s_tile;
-  __shared__ uint32_t s_off[FIRST ? OFF_CACHE : 1];
 
   // An id range error was latched before this launch (by the histogram):
   // every tile of every pass skips, consistently.
-  if (ld_volatile_u32(err.step) & ERR_ID_RANGE) return;
+  if (__syncthreads_or((ld_volatile_u32(err.step) & ERR_ID_RANGE) != 0u)) return;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   if (tid == 0) s_tile = atomicAdd(sc.tile_counter + pass, 1u);
   for (int i = tid; i < SORT_WARPS * RADIX; i += SORT_THREADS) (&s_warp[0][0])[i] = 0u;
   __syncthreads();
 
-  const uint32_t* offs = FIRST ? cache_offsets(a, s_off) : nullptr;
   const uint32_t tile = s_tile;
   const int64_t N = a.N;
   const int64_t base = (int64_t)tile * SORT_TILE;
@@ -224,8 +226,8 @@ __global__ void __launch_bounds__(SORT_THREADS)
   for (int j = 0; j < SORT_ITEMS; ++j) {
     const int64_t idx = base + (int64_t)warp * (SORT_ITEMS * 32) + j * 32 + lane;
     if (idx < N) {
-      if (FIRST) {
-        key[j] = occurrence_key(a, offs, idx, err);
+      if (FIRST) {  // keys written by the histogram kernel; payload = occurrence
+        key[j] = keys_in[idx];
         val[j] = (uint32_t)idx;
       } else {
         key[j] = keys_in[idx];
@@ -346,9 +348,9 @@ void launch_weights(const StepArgs& a, StepScratch sc, DevStats* stats, int n_hi
   k_message_weights<<<1, 256, 0, s>>>(a, sc, stats, n_hist_words);
 }
 
-void launch_sort_histogram(const StepArgs& a, int passes, StepScratch sc, ErrSink err, int grid,
-                           cudaStream_t s) {
-  k_sort_histogram<<<grid, SORT_THREADS, 0, s>>>(a, passes, sc, err);
+void launch_sort_histogram(const StepArgs& a, int passes, StepScratch sc, uint32_t* keys0,
+                           ErrSink err, int grid, cudaStream_t s) {
+  k_sort_histogram<<<grid, SORT_THREADS, 0, s>>>(a, passes, sc, keys0, err);
 }
 
 void launch_onesweep(const StepArgs& a, bool first, int pass, const uint32_t* keys_in,
