@@ -128,8 +128,9 @@ KERNEL_SOURCES = {
 
 
 def measured_traffic(kernel, workload):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel's
-    source is unchanged since the capture."""
+    """DRAM bytes per global step of a kernel class (all its launches in one
+    step) from the committed ncu launch list, if the class's sources are
+    unchanged since the capture."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
@@ -138,7 +139,7 @@ def measured_traffic(kernel, workload):
     e = j.get(workload, {}).get(kernel)
     if not e or e.get("source_sha") != source_sha(KERNEL_SOURCES[kernel]):
         return None
-    return e.get("dram_bytes_per_launch")
+    return e.get("dram_bytes_per_step")
 
 
 def max_over_ranks(x: float, pg, device="cpu") -> float:
