@@ -6,7 +6,7 @@
 // weights and optimizer state are read and written once.
 //
 // Each persistent CTA walks an equal contiguous share of the parameters in
-// tiles of up to 1024.  A producer warp streams
+// tiles of up to 2048.  A producer warp streams
 // the tile's slice of every kept message into a ring of shared-memory stages
 // with 1-D bulk async copies (cp.async.bulk, completion counted on an mbarrier
 // per stage); eight consumer warps sum the slices with compensated (TwoSum)
@@ -21,9 +21,10 @@ namespace gba {
 
 namespace {
 
-constexpr int DT = 1024;           // parameters per tile
-constexpr int STAGES = 16;         // 4 KB each
-constexpr int CONSUMER_WARPS = 8;  // 256 threads, one float4 each
+constexpr int DT = 2048;           // parameters per tile
+constexpr int STAGES = 8;          // 8 KB each
+constexpr int CONSUMER_WARPS = 8;  // 256 threads, two float4 each
+constexpr int HALF = DT / 2;       // thread c owns [4c, 4c+4) and [HALF+4c, HALF+4c+4)
 constexpr int DENSE_THREADS = (CONSUMER_WARPS + 1) * 32;
 
 __global__ void __launch_bounds__(DENSE_THREADS)
@@ -87,23 +88,31 @@ __global__ void __launch_bounds__(DENSE_THREADS)
       }
     }
   } else {
-    // ---- consumers: thread c owns parameters [4c, 4c + 4) of each tile
+    // ---- consumers: thread c owns parameters [4c, 4c + 4) and
+    // [HALF + 4c, HALF + 4c + 4) of each tile
     const int c = tid;
     const float Mf = (float)da.M;
     uint32_t q = 0;
     for (int64_t start = r0; start < r1; start += DT) {
       const int64_t n = r1 - start < DT ? r1 - start : DT;
-      const bool mine = (int64_t)c * 4 < n;
-      const int64_t e = start + (int64_t)c * 4;
-      float4 w = make_float4(0.f, 0.f, 0.f, 0.f), s0 = w, s1 = w;
-      if (mine) {
-        w = *reinterpret_cast<const float4*>(da.w + e);
-        s0 = *reinterpret_cast<const float4*>(da.s0 + e);
-        if (da.opt.kind == 1) s1 = *reinterpret_cast<const float4*>(da.s1 + e);
-      }
-      CSum acc[4];
+      bool mine[2];
+      int64_t e[2];
+      float4 w[2], s0[2], s1[2];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) acc[i] = CSum{0.f, 0.f};
+      for (int h = 0; h < 2; ++h) {
+        const int64_t off = (int64_t)h * HALF + (int64_t)c * 4;
+        mine[h] = off < n;
+        e[h] = start + off;
+        w[h] = s0[h] = s1[h] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (mine[h]) {
+          w[h] = *reinterpret_cast<const float4*>(da.w + e[h]);
+          s0[h] = *reinterpret_cast<const float4*>(da.s0 + e[h]);
+          if (da.opt.kind == 1) s1[h] = *reinterpret_cast<const float4*>(da.s1 + e[h]);
+        }
+      }
+      CSum acc[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = CSum{0.f, 0.f};
       bool aborted = false;
       for (int j = 0; j < n_kept; ++j, ++q) {
         const int stage = (int)(q % STAGES);
@@ -119,27 +128,34 @@ __global__ void __launch_bounds__(DENSE_THREADS)
           aborted = true;
           break;
         }
-        if (mine) {
-          const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT + 4 * c);
-          csum_add(acc[0], v.x);
-          csum_add(acc[1], v.y);
-          csum_add(acc[2], v.z);
-          csum_add(acc[3], v.w);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          if (mine[h]) {
+            const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT +
+                                                              h * HALF + 4 * c);
+            csum_add(acc[4 * h + 0], v.x);
+            csum_add(acc[4 * h + 1], v.y);
+            csum_add(acc[4 * h + 2], v.z);
+            csum_add(acc[4 * h + 3], v.w);
+          }
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(empty + stage);
       }
       if (aborted || __shfl_sync(0xffffffffu, *(volatile int*)&s_abort, 0) != 0) break;
-      if (mine) {
-        float wv[4] = {w.x, w.y, w.z, w.w}, a0[4] = {s0.x, s0.y, s0.z, s0.w},
-              a1[4] = {s1.x, s1.y, s1.z, s1.w};
 #pragma unroll
-        for (int i = 0; i < 4; ++i) opt_update(da.opt, wv[i], a0[i], a1[i],
-                                               __fdiv_rn(csum_value(acc[i]), Mf));
-        *reinterpret_cast<float4*>(da.w + e) = make_float4(wv[0], wv[1], wv[2], wv[3]);
-        *reinterpret_cast<float4*>(da.s0 + e) = make_float4(a0[0], a0[1], a0[2], a0[3]);
+      for (int h = 0; h < 2; ++h) {
+        if (!mine[h]) continue;
+        float wv[4] = {w[h].x, w[h].y, w[h].z, w[h].w},
+              a0[4] = {s0[h].x, s0[h].y, s0[h].z, s0[h].w},
+              a1[4] = {s1[h].x, s1[h].y, s1[h].z, s1[h].w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          opt_update(da.opt, wv[i], a0[i], a1[i], __fdiv_rn(csum_value(acc[4 * h + i]), Mf));
+        *reinterpret_cast<float4*>(da.w + e[h]) = make_float4(wv[0], wv[1], wv[2], wv[3]);
+        *reinterpret_cast<float4*>(da.s0 + e[h]) = make_float4(a0[0], a0[1], a0[2], a0[3]);
         if (da.opt.kind == 1)
-          *reinterpret_cast<float4*>(da.s1 + e) = make_float4(a1[0], a1[1], a1[2], a1[3]);
+          *reinterpret_cast<float4*>(da.s1 + e[h]) = make_float4(a1[0], a1[1], a1[2], a1[3]);
       }
     }
     // The last (D mod 4) parameters: plain loads, CTA 0.
