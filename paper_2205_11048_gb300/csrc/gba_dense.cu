@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
       for (int j = 0; j < n_kept; ++j, ++q) {
         const int stage = (int)(q % STAGES);
         const uint32_t ph = (q / STAGES) & 1u;
-        // Every lane waits (acquiring the copied bytes); the verdict is made
+        // Every lane waits (acquiring the copied bytes); the outcome is made
         // warp-uniform so the warp leaves the loop together.
         const bool ok = __all_sync(0xffffffffu, mbar_wait(full + stage, ph, wait_ns));
         if (!ok) {

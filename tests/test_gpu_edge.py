@@ -186,8 +186,8 @@ def test_varying_local_batches_overshoot():
 
 
 def test_hot_row_spanning_many_warps():
-    """One row with 200K occurrences in a step: partial sums cross many warp
-    ranges and are stitched by the fixup kernel in order."""
+    """One row with 200K occurrences in a step: its partial sums span hundreds
+    of reduction windows and are merged by the cross-window kernel."""
     gen = torch.Generator(device="cuda").manual_seed(1)
     cfg = cfg_of([(5000, 16, 0, 1)], D=4, G=4, iota=2)
     steps = []
