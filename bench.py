@@ -245,7 +245,6 @@ def run_gba(args):
 
     from paper_2205_11048_gb300 import binding as B
     from paper_2205_11048_gb300 import workload as W
-    from tests import _harness as H
 
     ws, rank, local = dist_setup()
     torch.cuda.set_device(local)
@@ -270,7 +269,7 @@ def run_gba(args):
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
     # consecutive steps overlap (step k+1's sort during step k's row update)
-    g = H.make_gpu(cfg, max_buf=2 * M, debug=False, overlap=True)
+    g = B.gba_for_workload(cfg, max_buf=2 * M, overlap=True)
     # pre-built ctypes arguments for the by-reference pushes
     pre = []
     for b in batches:
@@ -365,7 +364,7 @@ def run_gba(args):
             host.append(hb)
         h2d = sum(sum(x.numel() * 8 for x in m["ids"]) + sum(x.numel() * 4 for x in m["rows"])
                   + m["dense"].numel() * 4 for m in host[0])
-        g2 = H.make_gpu(cfg, max_buf=2 * M, debug=False)
+        g2 = B.gba_for_workload(cfg, max_buf=2 * M)
         pre2 = []
         for hb in host:
             row = []

@@ -195,6 +195,22 @@ def opt_desc(kind=ADAGRAD, lr=0.01, init_acc=0.1, beta1=0.9, beta2=0.999, eps=1e
     return gba_opt_desc(kind, lr, init_acc, beta1, beta2, eps)
 
 
+def gba_for_workload(cfg, max_buf=None, seed=None, overlap=False, **rule):
+    """A handle sized for a workload description (a `workload.WorkloadCfg`:
+    tables, dense size, optimizers, global batch, tolerance iota), with room
+    for max_buf buffered messages (default two global batches)."""
+    def od(o):
+        return opt_desc(o.kind, o.lr, o.init_acc, o.beta1, o.beta2, o.eps)
+    tables = [(tb.rows, tb.dim, tb.id_mode, cfg.max_ids_per_msg(t), od(tb.opt))
+              for t, tb in enumerate(cfg.tables)]
+    rule = rule or dict(iota=cfg.iota)
+    g = GBA(tables, cfg.D, od(cfg.dense_opt), cfg.G, max_buf or 2 * cfg.M,
+            seed=cfg.seed if seed is None else seed, **rule)
+    if overlap:
+        g.set_overlap(True)
+    return g
+
+
 class GBA:
     """One parameter-server state on the current CUDA device."""
 

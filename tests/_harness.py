@@ -23,15 +23,9 @@ def opt_desc(o: W.OptCfg):
 
 
 def make_gpu(cfg: W.WorkloadCfg, max_buf=None, seed=None, debug=True, rule=None, overlap=False):
-    tables = [(tb.rows, tb.dim, tb.id_mode, cfg.max_ids_per_msg(t), opt_desc(tb.opt))
-              for t, tb in enumerate(cfg.tables)]
-    rule = rule or dict(iota=cfg.iota)
-    g = B.GBA(tables, cfg.D, opt_desc(cfg.dense_opt), cfg.G, max_buf or 2 * cfg.M,
-              seed=cfg.seed if seed is None else seed, **rule)
+    g = B.gba_for_workload(cfg, max_buf=max_buf, seed=seed, overlap=overlap, **(rule or {}))
     if debug:
         g.set_debug(True)
-    if overlap:
-        g.set_overlap(True)
     return g
 
 
