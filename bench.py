@@ -50,7 +50,11 @@ def alg_bytes(cfg, st_delta, steps):
     """Algorithmic bytes per step by kernel (the bytes the method must move):
     ids 8 B per occurrence (sort), kept gradient rows 4d B, per applied row its
     state read + written (2 * S_opt * 4d B) and tag (8 B), dense: kept messages'
-    gradients 4D B each plus the dense state read + written (2 * S_opt * 4D)."""
+    gradients 4D B each plus the dense state read + written (2 * S_opt * 4D).
+    The tables of every workload here share one width and optimizer; the
+    counters are summed over tables."""
+    assert all(t.dim == cfg.tables[0].dim and t.opt.kind == cfg.tables[0].opt.kind
+               for t in cfg.tables), "tables of different widths or optimizers"
     tb = cfg.tables[0]
     d = tb.dim
     s_opt_rows = 2 if tb.opt.kind == 0 else 3
