@@ -70,6 +70,48 @@ def pin_hand_adagrad(L):
             assert orc.last_stats[key] == val, ("stats", key, orc.last_stats[key], val)
 
 
+def _check_hand_step(orc, tb, e, w0, dw0):
+    assert orc.last_keep.tolist() == e["keep"], ("keep", orc.last_keep)
+    cnt = orc.last_count[0]
+    kept = orc.last_kept[0]
+    touched = np.nonzero(cnt)[0].tolist()
+    assert touched == e["touched"], ("touched", touched)
+    assert cnt[touched].tolist() == e["count"], ("count", cnt)
+    assert kept[touched].tolist() == e["kept"], ("kept", kept)
+    w = orc.tables[0].w.astype(np.float64).reshape(tb.rows, tb.dim)
+    acc = orc.tables[0].s0.reshape(tb.rows, tb.dim)
+    for r in range(tb.rows):
+        assert (w[r] - w0[r]).tolist() == [F(v) for v in e["dw"][str(r)]], \
+            ("dw", r, (w[r] - w0[r]).tolist())
+        assert acc[r].astype(np.float64).tolist() == [F(v) for v in e["acc"][str(r)]], ("acc", r)
+    assert orc.tables[0].ver.tolist() == e["ver"], ("ver", orc.tables[0].ver)
+    dw = (orc.dense.w.astype(np.float64) - dw0).tolist()
+    assert dw == [F(v) for v in e["dense_dw"]], ("dense dw", dw)
+    assert orc.dense.s0.astype(np.float64).tolist() == [F(v) for v in e["dense_acc"]]
+    for key, val in e["stats"].items():
+        assert orc.last_stats[key] == val, ("stats", key, orc.last_stats[key], val)
+
+
+def pin_hand_rule_options(L):
+    """Hand-worked steps of the optional readings: a row's sum divided by its
+    kept messages, or by M; rows decayed by the message staleness k - token."""
+    g = load_golden()["rule_options"]
+    for var in g["variants"]:
+        tb = O.TableSpec(g["table"]["rows"], g["table"]["dim"],
+                         O.OptSpec(O.ADAGRAD, F(g["table"]["lr"]), F(g["table"]["init_acc"])))
+        dopt = O.OptSpec(O.ADAGRAD, F(g["dense"]["lr"]), F(g["dense"]["init_acc"]))
+        orc = O.OracleGBA([tb], g["dense"]["D"], dopt, g["global_batch"], seed=4321, library=L,
+                          **var["rule"])
+        w0 = orc.tables[0].w.astype(np.float64).reshape(tb.rows, tb.dim).copy()
+        dw0 = orc.dense.w.astype(np.float64).copy()
+        for step in (g["step0"], var["step1"]):
+            assert orc.pull_version() == step["k"]
+            for m in step["messages"]:
+                orc.push(_msg(m))
+            assert orc.try_apply() == 1
+            _check_hand_step(orc, tb, step["expect"], w0, dw0)
+
+
 def pin_hand_adam(L):
     """One textbook Adam step with dyadic hyper-parameters."""
     g = load_golden()["adam"]
@@ -368,8 +410,8 @@ def pin_brute_force(L, seed=21):
         assert orc.dense.s0.tolist() == [float(v) for v in DS0]
 
 
-ALL_PINS = [pin_hand_adagrad, pin_hand_adam, pin_sync_closed_form, pin_decay_boundary,
-            pin_fifo_prefix, pin_order_invariance, pin_brute_force]
+ALL_PINS = [pin_hand_adagrad, pin_hand_rule_options, pin_hand_adam, pin_sync_closed_form,
+            pin_decay_boundary, pin_fifo_prefix, pin_order_invariance, pin_brute_force]
 
 
 def pin_init_published(L):

@@ -35,6 +35,19 @@ MUTATIONS = [
      "S += (double)dense_grads[m][e];", 0),
     ("init-scale", "return (float)top * 0x1p-27f;", "return (float)top * 0x1p-26f;", 0),
     ("fifo-overshoot", "if (acc >= G) return i + 1;", "if (acc > G) return i + 1;", 0),
+    # the optional readings (kept-message and M denominators, message staleness for rows)
+    ("kept-denominator-counts-all", "if (rule->sparse_denominator == 1) denom = cnt_kept[r];",
+     "if (rule->sparse_denominator == 1) denom = cnt[r];", 0),
+    ("kept-denominator-counts-occurrences", "if (rule->sparse_denominator == 1) denom = cnt_kept[r];",
+     "if (rule->sparse_denominator == 1) denom = kept_occ[r];", 0),
+    ("m-denominator-counts-all", "if (rule->sparse_denominator == 2) denom = M;",
+     "if (rule->sparse_denominator == 2) denom = cnt[r];", 0),
+    ("m-denominator-counts-kept", "if (rule->sparse_denominator == 2) denom = M;",
+     "if (rule->sparse_denominator == 2) denom = st.msgs_kept;", 0),
+    ("message-staleness-option-ignored", "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k;",
+     "int64_t ref = tb->ver[r];", 0),
+    ("message-staleness-off-by-one", "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k;",
+     "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k + 1;", 0),
 ]
 
 
