@@ -4,14 +4,18 @@ One "step" is one global step of the hot path: message weights (Eq. (1)),
 the radix sort + dedup of the global batch's ids, the per-row decayed
 segment-sum and row update, and the dense reduce + optimizer.
 
-Default workload: the 32-worker one-hot workload (1e7 x 32 embedding table,
-Adagrad; 1M dense parameters, Adam; 32 messages of local batch 1024, 26 ids per
-sample; geometric staleness with 10% stragglers).  Inputs are synthetic
-(seeded Zipf ids, N(0, 0.01^2) gradients) and resident in HBM before the timed
-region; messages are pushed by reference, R distinct global batches in turn,
-with fresh tokens every step.
+Default workload: the largest single-GPU one -- 128 workers of local batch
+1024 (global batch 131,072), one 2e8 x 64 embedding table of hashed 64-bit ids
+(MODULO rows) with its Adagrad accumulator, 40 one-hot Zipf(1.05) fields, 8M
+dense parameters with Adam, geometric staleness (mean 3) with 20% stragglers.
+Inputs are synthetic (seeded Zipf ids, N(0, 0.01^2) gradients) and resident in
+HBM before the timed region; messages are pushed by reference, two distinct
+global batches in turn (each larger than the 129 MB L2), with fresh tokens
+every step.  The timed region ends with the library's streams joined into the
+timing stream, so it covers all of the steps' work.
 
-Prints one JSON line (rank 0).  --impl reference times the CPU oracle instead.
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle instead,
+on the same workload description.
 """
 from __future__ import annotations
 
@@ -29,7 +33,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "global-batch aggregate+apply steps/s; applied grad rows/s; HBM GB/s vs ~8 TB/s peak"
-R_BATCHES = 4
+R_BATCHES = 2
 
 
 def peaks():
@@ -168,51 +172,81 @@ def dist_setup():
     return ws, rank, local
 
 
-def run_reference(args):
-    """The CPU oracle, as it stands, on this host's cores, same workload."""
-    ws, rank, _ = dist_setup()
-    if rank != 0:
-        return
-    import numpy as np
-    import torch
+def config_dict(cfg, ws):
+    """The workload description both arms print (the same dict in each)."""
+    in_bytes = cfg.M * (sum(cfg.ids_per_msg(t) * (8 + 4 * tb.dim)
+                            for t, tb in enumerate(cfg.tables)) + 4 * cfg.D)
+    return {"workload": cfg.name, "M": cfg.M, "B": cfg.B, "G": cfg.G,
+            "tables": [[t.rows, t.dim] for t in cfg.tables], "dense": cfg.D,
+            "iota": cfg.iota, "batches_in_turn": R_BATCHES,
+            "l2": f"inputs larger than L2: each global batch holds {in_bytes / 1e6:.0f} MB of "
+                  f"ids and gradients, {R_BATCHES} distinct batches in turn",
+            "parallelism": f"replicas x{ws}"}
 
-    from oracle import oracle as O
+
+def touched_rows(cfg, batches_cpu):
+    """Per table, the sorted rows that the batches' ids map to."""
+    import numpy as np
+    from tests import _harness as H
+    out = []
+    for t in range(len(cfg.tables)):
+        rows = [H.rows_of(cfg, t, m["ids"][t].numpy()) for b in batches_cpu for m in b]
+        out.append(np.unique(np.concatenate(rows)) if rows else np.zeros(0, np.int64))
+    return out
+
+
+def oracle_rate(cfg, batches_cpu, warmup, steps):
+    """The CPU oracle, as it stands, one thread: full global steps of the
+    workload on the given batches (in turn, tokens drawn per step as on the
+    GPU).  It holds every dense parameter and every row the batches touch;
+    rows are independent of one another, so this is the full model restricted
+    to the state these steps read and write.  State initialisation is outside
+    the timed part.  Returns (steps/s, description of the sample)."""
     from paper_2205_11048_gb300 import workload as W
     from tests import _harness as H
-    cfg = workload_cfg(args.config)
-    batches = [W.generate_step(cfg, r, "cpu") for r in range(R_BATCHES)]
-    orc_msgs = [[H.to_oracle(m) for m in b] for b in batches]
+    track = touched_rows(cfg, batches_cpu)
+    orc_msgs = [[H.to_oracle(m) for m in b] for b in batches_cpu]
     t0 = time.perf_counter()
-    orc = H.make_oracle(cfg)
+    orc = H.make_oracle(cfg, track_rows=track)
     setup_s = time.perf_counter() - t0
-    budget = args.ref_budget_s
 
     def step(k):
-        toks = W.tokens_for_step(cfg, k)
-        for m, tok in zip(orc_msgs[k % R_BATCHES], toks):
+        for m, tok in zip(orc_msgs[k % len(orc_msgs)], W.tokens_for_step(cfg, k)):
             m.token = tok
             orc.push(m)
         assert orc.try_apply() == 1
 
     k = 0
-    for _ in range(max(0, min(args.warmup, 3))):
+    for _ in range(warmup):
         step(k)
         k += 1
     t0 = time.perf_counter()
-    n = 0
-    while n < args.steps and (time.perf_counter() - t0) < budget:
+    for _ in range(steps):
         step(k)
         k += 1
-        n += 1
     el = time.perf_counter() - t0
-    sps = n / el
-    sample = (f"{n} full global steps of {cfg.name} (all {cfg.tables[0].rows} rows and "
-              f"{cfg.D} dense parameters tracked), single thread, {R_BATCHES} distinct "
-              f"batches in turn; state init {setup_s:.1f} s excluded")
-    line = {"impl": "reference", "metric": METRIC, "value": sps, "unit": "steps/s", "n_gpus": ws,
-            "steps": n, "warmup": min(args.warmup, 3), "ms_per_step": 1e3 * el / max(n, 1),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-            "data": "synthetic", "config": {"workload": cfg.name, "M": cfg.M, "B": cfg.B},
+    n_rows = sum(len(t) for t in track)
+    sample = (f"{steps} full global steps of {cfg.name} after {warmup} warm-up steps, one "
+              f"thread, {len(batches_cpu)} distinct batches in turn; state of all {cfg.D} "
+              f"dense parameters and the {n_rows} rows the batches touch, initialised in "
+              f"{setup_s:.1f} s outside the timing; {el:.1f} s timed")
+    return steps / el, sample
+
+
+def run_reference(args):
+    """The CPU oracle on this host's cores, same workload, warm-up and steps."""
+    ws, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    from paper_2205_11048_gb300 import workload as W
+    cfg = workload_cfg(args.config)
+    batches = [W.generate_step(cfg, r, "cpu") for r in range(R_BATCHES)]
+    sps, sample = oracle_rate(cfg, batches, args.warmup, args.steps)
+    line = {"impl": "reference", "metric": METRIC, "value": sps, "unit": "steps/s",
+            "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 / sps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded Zipf ids, "
+            "N(0,0.01^2) grads; generated on the host)", "config": config_dict(cfg, ws),
             "cpu_baseline": {"value": sps, "unit": "steps/s", "cores": 1, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": sps, "unit": "steps/s", "h2d_bytes_per_step": 0,
@@ -220,31 +254,18 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def cpu_baseline(cfg, batches_cpu, budget_s):
-    """Oracle steps/s on this host, one thread, on the same batches."""
-    from paper_2205_11048_gb300 import workload as W
-    from tests import _harness as H
-    orc_msgs = [[H.to_oracle(m) for m in b] for b in batches_cpu]
-    orc = H.make_oracle(cfg)
-    t0 = time.perf_counter()
-    n = 0
-    k = 0
-    while time.perf_counter() - t0 < budget_s:
-        toks = W.tokens_for_step(cfg, k)
-        for m, tok in zip(orc_msgs[k % len(orc_msgs)], toks):
-            m.token = tok
-            orc.push(m)
-        orc.try_apply()
-        n += 1
-        k += 1
-    el = time.perf_counter() - t0
-    return {"value": n / el, "unit": "steps/s", "cores": 1, "kind": "oracle",
-            "sample": f"{n} full global steps of {cfg.name} on the CPU oracle, one thread, "
-                      f"{el:.1f} s"}
+def push_args(B, cfg, batch):
+    """ctypes arguments of gba_push / gba_push_ref for every message of a batch."""
+    out = []
+    for m in batch:
+        grads = (B.gba_sparse_grad * max(1, len(cfg.tables)))(*[
+            B.gba_sparse_grad(m["ids"][t].data_ptr(), m["ids"][t].numel(),
+                              m["rows"][t].data_ptr()) for t in range(len(cfg.tables))])
+        out.append((grads, ctypes.c_void_p(m["dense"].data_ptr()), m["local_batch"]))
+    return out
 
 
 def run_gba(args):
-    import numpy as np
     import torch
 
     from paper_2205_11048_gb300 import binding as B
@@ -274,45 +295,30 @@ def run_gba(args):
     stream = torch.cuda.current_stream()
     # consecutive steps overlap (step k+1's sort during step k's row update)
     g = B.gba_for_workload(cfg, max_buf=2 * M, overlap=True)
-    # pre-built ctypes arguments for the by-reference pushes
-    pre = []
-    for b in batches:
-        row = []
-        for m in b:
-            grads = (B.gba_sparse_grad * len(cfg.tables))(*[
-                B.gba_sparse_grad(m["ids"][t].data_ptr(), m["ids"][t].numel(),
-                                  m["rows"][t].data_ptr()) for t in range(len(cfg.tables))])
-            row.append((grads, ctypes.c_void_p(m["dense"].data_ptr()), m["local_batch"]))
-        pre.append(row)
-    tokens = {}
+    pre = [push_args(B, cfg, b) for b in batches]
+    # tokens of every step this run applies, drawn before any timing
+    n_total = args.warmup + 2 * args.steps + (args.e2e_steps + 2 if args.e2e_steps > 0 else 0)
+    tokens = [W.tokens_for_step(cfg, k) for k in range(n_total)]
 
-    def toks(k):
-        if k not in tokens:
-            tokens[k] = W.tokens_for_step(cfg, k)
-        return tokens[k]
-
-    def step(k):
-        tk = toks(k)
-        for i, (grads, dense, b) in enumerate(pre[k % R_BATCHES]):
-            rc = L.gba_push_ref(g.h, tk[i], grads, dense, b)
+    def step(k, push=L.gba_push_ref, args_=pre):
+        tk = tokens[k]
+        for i, (grads, dense, b) in enumerate(args_[k % len(args_)]):
+            rc = push(g.h, tk[i], grads, dense, b)
             if rc != 0:
-                raise B.GBAError(rc, "push_ref")
+                raise B.GBAError(rc, "push")
         rc = L.gba_try_apply(g.h)
         if rc != 1:
             raise B.GBAError(rc, "try_apply")
 
-    n_total = args.warmup + args.steps
-    for k in range(n_total):
-        toks(k)
+    sampler = ClockSampler(local)
     k = 0
     for _ in range(args.warmup):
         step(k)
         k += 1
+    g.join()
     g.sync()
     st0 = g.stats()
-    g.set_timing(True)
-    sampler = ClockSampler(local)
-    time.sleep(0.3)
+    g.set_timing(False)  # clears the launch counters; no events inside the timed region
     if pg:
         pg.barrier()
     torch.cuda.synchronize()
@@ -322,95 +328,89 @@ def run_gba(args):
     for _ in range(args.steps):
         step(k)
         k += 1
+    g.join()  # the timing stream waits for every step's segment-sum, row and dense work
     ev1.record(stream)
     torch.cuda.synchronize()
     el_ms = ev0.elapsed_time(ev1)
     if pg:
         pg.barrier()
-    clocks = sampler.stop()
-    kt = g.kernel_times()
-    g.sync()
+    launches = sum(n for name, (n, _) in g.kernel_times().items() if name != "init")
     st1 = g.stats()
     delta = {key: st1[key] - st0[key] for key in st1}
     el_ms = max_over_ranks(el_ms, pg, "cuda")
     ms_per_step = el_ms / args.steps
     value = job_throughput(args.steps, ws, el_ms)
-    launches = sum(kt[n][0] for n in kt if n != "init")
+
+    # Per-kernel device times: a second pass of the same number of steps with
+    # every launch bracketed by events on its own stream (outside the timed
+    # region above; kernels of consecutive steps still run concurrently).
+    g.set_timing(True)
+    for _ in range(args.steps):
+        step(k)
+        k += 1
+    g.join()
+    kt = g.kernel_times()
+    g.set_timing(False)
+    clocks = sampler.stop()
 
     # roofline of the dominant kernel class: the one that must move the most
-    # algorithmic bytes (its time is measured live, concurrent steps included)
+    # algorithmic bytes
     bytes_, per = alg_bytes(cfg, delta, args.steps)
-    # the row path is three kernels per table (segment reduction, rows that
-    # cross windows, row update): its bytes are divided by their summed time
-    classes = {"rows": kt["seg_reduce"][1] + kt["seg_cross"][1] + kt["row_update"][1],
+    classes = {"rows": kt["seg_scan"][1] + kt["row_long"][1] + kt["row_apply"][1],
                "dense": kt["dense"][1], "sort": kt["sort_hist"][1] + kt["sort_pass"][1]}
-    dom = max(("rows", "dense", "sort"), key=lambda c: bytes_[c])
-    n_launch = {"rows": kt["seg_reduce"][0] + kt["seg_cross"][0] + kt["row_update"][0],
+    n_launch = {"rows": kt["seg_scan"][0] + kt["row_long"][0] + kt["row_apply"][0],
                 "dense": kt["dense"][0], "sort": kt["sort_hist"][0] + kt["sort_pass"][0]}
+    dom = max(("rows", "dense", "sort"), key=lambda c: bytes_[c])
     launches_per_step = max(1, n_launch[dom] // args.steps)
     dur_ms = classes[dom] / args.steps  # one step's launches of that class
     peak, peak_kind = peaks()
     achieved = bytes_[dom] / (dur_ms / 1e3) / 1e9
     traffic = measured_traffic(dom, cfg.name)
 
-    # end to end through the C ABI with host buffers: pinned host -> device
-    # copies inside gba_push, one step, and a device -> host read of the counters
+    # End to end through the C ABI with host buffers: every step copies its M
+    # messages from pinned host memory (gba_push) and reads the step's counters
+    # back (gba_stats), on the same handle with steps no longer overlapping.
     e2e = None
     if args.e2e_steps > 0:
-        host = []
-        for b in batches[:2]:
-            hb = []
-            for m in b:
-                hb.append(dict(token=0, local_batch=m["local_batch"],
-                               ids=[x.cpu().pin_memory() for x in m["ids"]],
-                               rows=[x.cpu().pin_memory() for x in m["rows"]],
-                               dense=m["dense"].cpu().pin_memory()))
-            host.append(hb)
+        g.set_overlap(False)
+        hb = [dict(local_batch=m["local_batch"],
+                   ids=[x.cpu().pin_memory() for x in m["ids"]],
+                   rows=[x.cpu().pin_memory() for x in m["rows"]],
+                   dense=m["dense"].cpu().pin_memory()) for m in batches[0]]
         h2d = sum(sum(x.numel() * 8 for x in m["ids"]) + sum(x.numel() * 4 for x in m["rows"])
-                  + m["dense"].numel() * 4 for m in host[0])
-        g2 = B.gba_for_workload(cfg, max_buf=2 * M)
-        pre2 = []
-        for hb in host:
-            row = []
-            for m in hb:
-                grads = (B.gba_sparse_grad * len(cfg.tables))(*[
-                    B.gba_sparse_grad(m["ids"][t].data_ptr(), m["ids"][t].numel(),
-                                      m["rows"][t].data_ptr()) for t in range(len(cfg.tables))])
-                row.append((grads, ctypes.c_void_p(m["dense"].data_ptr()), m["local_batch"]))
-            pre2.append(row)
+                  + m["dense"].numel() * 4 for m in hb)
+        pre_host = [push_args(B, cfg, hb)]
         stats_out = B.gba_stats_t()
 
         def e2e_step(kk):
-            tk = toks(kk % n_total)
-            for i, (grads, dense, b) in enumerate(pre2[kk % 2]):
-                rc = L.gba_push(g2.h, tk[i], grads, dense, b)
-                if rc != 0:
-                    raise B.GBAError(rc, "push")
-            rc = L.gba_try_apply(g2.h)
-            if rc != 1:
-                raise B.GBAError(rc, "try_apply")
-            rc = L.gba_stats(g2.h, ctypes.byref(stats_out))  # reads the step's counters
+            step(kk, push=L.gba_push, args_=pre_host)
+            rc = L.gba_stats(g.h, ctypes.byref(stats_out))  # reads the step's counters
             if rc != 0:
                 raise B.GBAError(rc, "stats")
 
-        for kk in range(3):
-            e2e_step(kk)
+        for _ in range(2):
+            e2e_step(k)
+            k += 1
         torch.cuda.synchronize()
         t0 = time.perf_counter()
-        for kk in range(args.e2e_steps):
-            e2e_step(3 + kk)
+        for _ in range(args.e2e_steps):
+            e2e_step(k)
+            k += 1
         torch.cuda.synchronize()
         el = time.perf_counter() - t0
+        el = max_over_ranks(el, pg, "cuda")
         e2e = {"value": ws * args.e2e_steps / el, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": ctypes.sizeof(B.gba_stats_t), "steps": args.e2e_steps}
-        g2.close()
+        del hb, pre_host
 
     cpu = None
-    if rank == 0 and ws == 1 and args.cpu_budget_s > 0:
+    if rank == 0 and ws == 1 and args.cpu_steps > 0:
         cpu_batches = [[{"token": m["token"], "local_batch": m["local_batch"],
                          "ids": [x.cpu() for x in m["ids"]], "rows": [x.cpu() for x in m["rows"]],
                          "dense": m["dense"].cpu()} for m in b] for b in batches]
-        cpu = cpu_baseline(cfg, cpu_batches, args.cpu_budget_s)
+        sps, sample = oracle_rate(cfg, cpu_batches, 1, args.cpu_steps)
+        cpu = {"value": sps, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": sample}
+        del cpu_batches
 
     if rank == 0:
         line = {
@@ -418,22 +418,20 @@ def run_gba(args):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded Zipf ids, N(0,0.01^2) grads; replicas per GPU)",
-            "config": {"workload": cfg.name, "M": cfg.M, "B": cfg.B, "G": cfg.G,
-                       "tables": [[t.rows, t.dim] for t in cfg.tables], "dense": cfg.D,
-                       "iota": cfg.iota, "batches_in_turn": R_BATCHES,
-                       "l2": "inputs larger than L2 (distinct global batches of "
-                             f"{bytes_['total'] / 1e6:.0f} MB of algorithmic traffic each)",
-                       "parallelism": f"replicas x{ws}"},
+            "config": config_dict(cfg, ws),
             "rows_per_s": per["occ"] * value,
             "unique_rows_per_s": per["u_touched"] * value,
             "alg_bytes_per_step": bytes_["total"],
             "alg_gbs": bytes_["total"] * value / ws / 1e9,
             "hbm_frac_of_8tbs": bytes_["total"] * value / ws / 8e12,
+            "hbm_frac_of_measured": bytes_["total"] * value / ws / 1e9 / peak,
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic, "alg_bytes_per_launch": bytes_[dom] / launches_per_step,
                          "launches_per_step": launches_per_step,
-                         "ms_per_step_in_kernel": dur_ms},
+                         "ms_per_step_in_kernel": dur_ms,
+                         "timing": "CUDA events around each launch on its stream, in a second "
+                                   "pass of the same steps after the timed region"},
             "kernels_ms_per_step": {n: kt[n][1] / args.steps for n in kt if n != "init"},
             "per_step": per,
             "clocks": clocks,
@@ -451,13 +449,14 @@ def run_gba(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=300)
-    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gba", choices=["gba", "reference"])
-    ap.add_argument("--config", type=int, default=2)
-    ap.add_argument("--e2e-steps", type=int, default=20)
-    ap.add_argument("--cpu-budget-s", type=float, default=15.0)
-    ap.add_argument("--ref-budget-s", type=float, default=60.0)
+    ap.add_argument("--config", type=int, default=5,
+                    help="workload 1-5 (default 5: the largest one that fits one GPU)")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--cpu-steps", type=int, default=3,
+                    help="oracle steps timed for the cpu_baseline leg (after one warm-up step)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -108,11 +108,12 @@ typedef struct {
 
 /* Per kernel class: launches and device time summed since timing was enabled. */
 /* indices into gba_kernel_times_t: K1 message weights; K2 sort (digit
- * histograms, one onesweep pass per key byte); K3 segment reduction, rows that
- * cross reduction windows, K4 row update; K5 dense update; table init. */
+ * histograms, one onesweep pass per key digit); K3 segment scan (decisions,
+ * row records, kept list); K3+K4 long rows (chunked sums and their update);
+ * K3+K4 row sums and update; K5 dense update; table init. */
 enum {
-  GBA_K_WEIGHTS = 0, GBA_K_SORT_HIST = 1, GBA_K_SORT_PASS = 2, GBA_K_SEG_REDUCE = 3,
-  GBA_K_SEG_CROSS = 4, GBA_K_ROW_UPDATE = 5, GBA_K_DENSE = 6, GBA_K_INIT = 7,
+  GBA_K_WEIGHTS = 0, GBA_K_SORT_HIST = 1, GBA_K_SORT_PASS = 2, GBA_K_SEG_SCAN = 3,
+  GBA_K_ROW_LONG = 4, GBA_K_ROW_APPLY = 5, GBA_K_DENSE = 6, GBA_K_INIT = 7,
   GBA_K_OTHER = 8, GBA_K_COUNT = 9
 };
 typedef struct {
@@ -179,8 +180,11 @@ gba_status gba_push_ref(gba_handle* h, int64_t token, const gba_sparse_grad* per
  */
 int32_t gba_try_apply(gba_handle* h);
 
-/* gba_pull_version - the number of global steps applied so far (k); a worker
- * that takes its token from here reports staleness k' - k when applied at k'. */
+/* gba_pull_version - the number of global steps applied so far (k).  Sec. 4.1
+ * defines a batch's token as the global step at which it is handed to a
+ * worker, and Alg. 2 (pull responding) hands the token out with the
+ * parameters; a worker that takes its token from here is counted as stale by
+ * k' - k when its gradient is applied at step k'.  NULL handle: -1. */
 int64_t gba_pull_version(gba_handle* h);
 
 /* gba_sync - wait for all work of the handle, then report any latched device error. */
@@ -212,6 +216,51 @@ void gba_destroy(gba_handle* h);
  * complete, in the handle's stream order, before later work on that stream.
  */
 gba_status gba_set_overlap(gba_handle* h, int32_t on);
+
+/*
+ * gba_pull - pull responding (Alg. 2: "look up the embedding tables based on
+ * the IDs for the embedding parameters" and send them to the worker).
+ *
+ * t      table index.
+ * ids    n device int64 ids (8-byte aligned), mapped to rows as in the table's
+ *        id_mode.
+ * out    n x dim device float32 (row-major), receives the rows' current
+ *        weights as of every step enqueued before this call.
+ * Enqueued on the handle's stream (after joining any overlapping steps); the
+ * rows are in out for work ordered after it on that stream.  A DIRECT id
+ * outside [0, rows) gets a row of zeros and is latched like a step's id error
+ * (the next gba_sync / gba_try_apply returns GBA_E_ID_RANGE).  GBA_E_ARG for a
+ * bad table index or NULL pointers with n > 0.
+ */
+gba_status gba_pull(gba_handle* h, int32_t t, const int64_t* ids, int64_t n, float* out);
+
+/*
+ * The token list (Sec. 4.1; Alg. 2 token generation and pull responding
+ * threads): a queue of tokens handed to workers with their batches.  Token
+ * values start at 0 and each repeats `repeats` (M) times, so the i-th token
+ * fetched is floor(i / M).  Whenever the queue holds fewer tokens than
+ * `workers`, new tokens are appended until it holds `workers` (the paper's
+ * refill, done under a lock).  gba_fetch_token may be called from any number
+ * of host threads at once.  The list needs no GPU.
+ *
+ * gba_token_list_create   GBA_E_ARG if repeats < 1 or workers < 1.
+ * gba_fetch_token         takes the head of the queue into *token.
+ * gba_token_list_state    tokens queued now, and fetched so far.
+ */
+typedef struct gba_token_list gba_token_list;
+gba_status gba_token_list_create(int64_t repeats, int32_t workers, gba_token_list** out);
+gba_status gba_fetch_token(gba_token_list* tl, int64_t* token);
+gba_status gba_token_list_state(gba_token_list* tl, int64_t* queued, int64_t* fetched);
+void gba_token_list_destroy(gba_token_list* tl);
+
+/*
+ * gba_join - order the handle's stream after every step enqueued so far (their
+ * segment-sum, row update and dense update included), without waiting on the
+ * host.  Work the caller enqueues on that stream afterwards, an event recorded
+ * there for instance, sees the results of every applied step.  Needed only
+ * with overlap on; with overlap off each gba_try_apply already does this.
+ */
+gba_status gba_join(gba_handle* h);
 
 /* ---- instrumentation and test entry points ----------------------------- */
 
@@ -258,14 +307,15 @@ gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream);
 /*
  * gba_sort_ids_static - sort one batch of ids by row without allocating.
  *
- * The paper has no counterpart to this entry point; it exists for callers that
- * cannot allocate device memory when they need the sort, for example code that
- * is being captured into a CUDA graph (an allocation is not a stream operation)
- * or a runtime whose device memory is entirely reserved up front.  It runs the
- * same histogram and onesweep radix-sort kernels as gba_try_apply, but takes
- * its scratch from one fixed device array of GBA_STATIC_SORT_BYTES bytes that
- * the library reserves when it is loaded; every GPU that loads the library
- * keeps that array until the process exits.  The call allocates nothing.
+ * The paper has no counterpart to this entry point.  It serves callers that
+ * must not allocate device memory at the moment they sort: a runtime that
+ * reserved all device memory up front and hands out no more, or an allocator's
+ * own hook, which cannot call back into cudaMalloc.  It runs the same
+ * histogram and onesweep radix-sort kernels as gba_try_apply, but takes its
+ * scratch from one fixed device array of GBA_STATIC_SORT_BYTES bytes that is
+ * part of the library image: every GPU that loads the library holds that array
+ * until the process exits.  The call itself allocates nothing (no cudaMalloc,
+ * cudaFree or allocating library routine).
  *
  * ids        n device int64 ids; row = id (id_mode DIRECT, 0 <= id < rows) or
  *            (uint64)id % rows (MODULO).
@@ -274,19 +324,31 @@ gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream);
  * rows_out   n device uint32: the rows of the ids in ascending order.
  * order_out  n device uint32: order_out[i] is the input index of rows_out[i];
  *            equal rows keep their input order (stable).
- * cuda_stream  the stream to run on (NULL: the legacy default stream); the call
- *            returns after the work has finished on it, with GBA_OK,
- *            GBA_E_ID_RANGE (a DIRECT id outside [0, rows)), GBA_E_DEVICE_TIMEOUT
- *            or GBA_E_CUDA.
+ * cuda_stream  the stream to run on (NULL: the legacy default stream).
+ *
+ * The call is synchronous: it enqueues its kernels on the stream, waits for the
+ * stream to finish, and returns GBA_OK, GBA_E_ID_RANGE (a DIRECT id outside
+ * [0, rows)), GBA_E_DEVICE_TIMEOUT (a bounded wait of the sort gave up) or
+ * GBA_E_CUDA (a CUDA call failed, or a CUDA error was already pending on the
+ * calling thread; a pending error is left in place for its owner).  It must
+ * not be called while the stream is being captured.  rows_out and order_out
+ * hold the sorted result only when GBA_OK is returned; after an error their
+ * contents are undefined.
  * The first call on a device, with that device current, looks up the array's
- * device address; make that first call before any stream capture.  All calls
- * share the one array and it keeps the previous call's contents (counters are
- * cleared at the start of each call); calls whose work overlaps on the GPU race.
+ * device address.  All calls share the one array, which keeps the previous
+ * call's contents (the counters that must start at zero are cleared at the
+ * start of each call): calls whose work overlaps on the GPU (two streams, or
+ * two host threads) race and give wrong results.
  */
 #define GBA_STATIC_SORT_MAX_IDS (1 << 20)
 #define GBA_STATIC_SORT_BYTES 9441392
 gba_status gba_sort_ids_static(const int64_t* ids, int64_t n, int64_t rows, int32_t id_mode,
                                uint32_t* rows_out, uint32_t* order_out, void* cuda_stream);
+
+/* gba_device_binary_version - the compute capability of the device code the
+ * library's kernels run from on the current device, as major * 10 + minor
+ * (103 for sm_103a), or GBA_E_CUDA when no device code could be loaded. */
+int32_t gba_device_binary_version(void);
 
 /* gba_version_string - library build identification. */
 const char* gba_version_string(void);

@@ -30,7 +30,7 @@ STATUS_NAMES = {0: "GBA_OK", -1: "GBA_E_ARG", -2: "GBA_E_ID_RANGE", -3: "GBA_E_O
 ADAGRAD, ADAM = 0, 1
 DIRECT, MODULO = 0, 1
 INT32_MAX = 2**31 - 1
-KERNEL_NAMES = ["weights", "sort_hist", "sort_pass", "seg_reduce", "seg_cross", "row_update",
+KERNEL_NAMES = ["weights", "sort_hist", "sort_pass", "seg_scan", "row_long", "row_apply",
                 "dense", "init", "other"]
 
 
@@ -99,6 +99,13 @@ _SIGNATURES = {
     "gba_kernel_times": (ctypes.c_int, [_P, ctypes.POINTER(gba_kernel_times_t)]),
     "gba_set_debug": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_set_overlap": (ctypes.c_int, [_P, ctypes.c_int32]),
+    "gba_join": (ctypes.c_int, [_P]),
+    "gba_pull": (ctypes.c_int, [_P, ctypes.c_int32, _P, ctypes.c_int64, _P]),
+    "gba_token_list_create": (ctypes.c_int, [ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(_P)]),
+    "gba_fetch_token": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int64)]),
+    "gba_token_list_state": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int64),
+                                            ctypes.POINTER(ctypes.c_int64)]),
+    "gba_token_list_destroy": (None, [_P]),
     "gba_debug_segments": (ctypes.c_int, [_P, ctypes.c_int64, _P, _P, _P, _P,
                                           ctypes.POINTER(ctypes.c_int64)]),
     "gba_debug_sorted": (ctypes.c_int, [_P, ctypes.c_int64, _P, _P,
@@ -107,6 +114,7 @@ _SIGNATURES = {
     "gba_debug_set_wait_limit": (ctypes.c_int, [_P, ctypes.c_int64]),
     "gba_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int64, _P]),
     "gba_version_string": (ctypes.c_char_p, []),
+    "gba_device_binary_version": (ctypes.c_int32, []),
     "gba_sort_ids_static": (ctypes.c_int, [_P, ctypes.c_int64, ctypes.c_int64, ctypes.c_int32,
                                            _P, _P, _P]),
 }
@@ -326,6 +334,20 @@ class GBA:
         check(self.L.gba_stats(self.h, ctypes.byref(s)), self.h)
         return s.as_dict()
 
+    def pull(self, t, ids):
+        """Current rows of table t for the device int64 tensor ids (pull responding)."""
+        torch = self.torch
+        ids = ids.contiguous()
+        out = torch.empty(ids.numel(), self.dims[t], dtype=torch.float32, device=ids.device)
+        check(self.L.gba_pull(self.h, int(t), ids.data_ptr() if ids.numel() else None,
+                              ids.numel(), out.data_ptr() if ids.numel() else None),
+              self.h, "gba_pull")
+        return out
+
+    def join(self):
+        """Order the handle's stream after every step enqueued so far."""
+        check(self.L.gba_join(self.h), self.h, "gba_join")
+
     def set_overlap(self, on=True):
         check(self.L.gba_set_overlap(self.h, int(on)), self.h)
 
@@ -399,3 +421,34 @@ def _gather_rows(ptr, rows, d, idx, dtype=None):
     elem = torch.empty((), dtype=dtype).element_size()
     raw = torch.as_tensor(_DevArray(ptr, rows * d * elem), device="cuda").view(dtype)
     return raw.view(rows, d).index_select(0, idx).clone()
+
+
+class TokenList:
+    """The token list of Sec. 4.1 / Alg. 2 (see gba_token_list_create)."""
+
+    def __init__(self, repeats, workers):
+        self.L = load()
+        self.h = _P()
+        check(self.L.gba_token_list_create(int(repeats), int(workers), ctypes.byref(self.h)),
+              what="gba_token_list_create")
+
+    def fetch(self):
+        t = ctypes.c_int64()
+        check(self.L.gba_fetch_token(self.h, ctypes.byref(t)), what="gba_fetch_token")
+        return int(t.value)
+
+    def state(self):
+        q, f = ctypes.c_int64(), ctypes.c_int64()
+        check(self.L.gba_token_list_state(self.h, ctypes.byref(q), ctypes.byref(f)))
+        return int(q.value), int(f.value)
+
+    def close(self):
+        if self.h:
+            self.L.gba_token_list_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

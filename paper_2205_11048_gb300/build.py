@@ -17,7 +17,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libgba.so")
 SOURCES = ["gba_host.cu", "gba_sort.cu", "gba_rows.cu", "gba_dense.cu", "gba_misc.cu",
-           "gba_noalloc.cu"]
+           "gba_noalloc.cu", "gba_pull.cu", "gba_tokens.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + os.path.join(ROOT, "include")]
 

@@ -127,22 +127,19 @@ struct gba_handle {
   unsigned long long* d_status[SLOTS] = {};
   int64_t status_tiles = 0;
   uint32_t epoch = 0;
-  uint32_t* d_dbg_count = nullptr;
-  uint32_t* d_dbg_kept = nullptr;
-  int64_t dbg_cap = 0;
   char* d_step_scratch[SLOTS] = {};
   StepScratch sc[SLOTS] = {};
-  // segment-sum and row-update buffers (apply stream only), grown with n_cap
-  RowDesc* d_desc = nullptr;
-  float* d_compact = nullptr;
-  float* d_rec_hi = nullptr;
-  float* d_rec_lo = nullptr;
-  uint32_t* d_rec_meta = nullptr;
-  unsigned long long* d_seg_status = nullptr;
-  uint32_t* d_seg_total = nullptr;
-  uint32_t* d_cross_list = nullptr;
-  uint32_t* d_cross_end = nullptr;
-  int64_t seg_win_cap = 0;
+  // row-kernel buffers (apply stream only), grown with n_cap
+  uint4* d_rr = nullptr;                   // row records, per table nbase[t] + t
+  const float** d_kl = nullptr;            // kept list, per table nbase[t]
+  float* d_kw = nullptr;                   // kept weights
+  unsigned long long* d_scan_status = nullptr;
+  uint4* d_long_rows = nullptr;
+  uint32_t* d_long_done = nullptr;
+  uint2* d_items = nullptr;
+  float* d_part_hi = nullptr;
+  float* d_part_lo = nullptr;
+  uint32_t* d_seg_total = nullptr;         // [T] rows of each table in the last step
   int d_max = 1;
 
   uint32_t* d_err = nullptr;
@@ -166,6 +163,7 @@ struct gba_handle {
   int last_buf = 0;
   int last_slot = 0;
   int32_t last_M = 0;
+  std::vector<int64_t> last_nbase;
 };
 
 namespace {
@@ -291,17 +289,10 @@ void free_all(gba_handle* h) {
     if (h->h_meta[i]) cudaFreeHost(h->h_meta[i]);
     if (h->meta_ev[i]) cudaEventDestroy(h->meta_ev[i]);
   }
-  cudaFree(h->d_dbg_count);
-  cudaFree(h->d_dbg_kept);
-  cudaFree(h->d_desc);
-  cudaFree(h->d_compact);
-  cudaFree(h->d_rec_hi);
-  cudaFree(h->d_rec_lo);
-  cudaFree(h->d_rec_meta);
-  cudaFree(h->d_seg_status);
-  cudaFree(h->d_seg_total);
-  cudaFree(h->d_cross_list);
-  cudaFree(h->d_cross_end);
+  for (void* p : {(void*)h->d_rr, (void*)h->d_kl, (void*)h->d_kw, (void*)h->d_scan_status,
+                  (void*)h->d_long_rows, (void*)h->d_long_done, (void*)h->d_items,
+                  (void*)h->d_part_hi, (void*)h->d_part_lo, (void*)h->d_seg_total})
+    cudaFree(p);
   cudaFree(h->d_err);
   if (h->h_err) cudaFreeHost(h->h_err);
   cudaFree(h->d_stats);
@@ -384,39 +375,34 @@ gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
     }
     h->n_cap = cap;
     h->status_tiles = tiles;
-    // segment buffers: one list entry (and compact row) per possible row head,
-    // records and look-back words per window
-    const int64_t cs = (h->d_max + 3) / 4 * 4;
-    const int64_t wins = seg_window_bound(cap, h->num_sms);
-    for (void* p : {(void*)h->d_desc, (void*)h->d_compact, (void*)h->d_rec_hi, (void*)h->d_rec_lo,
-                    (void*)h->d_rec_meta, (void*)h->d_seg_status, (void*)h->d_cross_list,
-                    (void*)h->d_cross_end})
+    // row-kernel buffers: a record per possible row (and one per table for the
+    // totals), a kept-list entry per occurrence, look-back words per scan tile,
+    // long rows and their chunks
+    for (void* p : {(void*)h->d_rr, (void*)h->d_kl, (void*)h->d_kw, (void*)h->d_scan_status,
+                    (void*)h->d_long_rows, (void*)h->d_long_done, (void*)h->d_items,
+                    (void*)h->d_part_hi, (void*)h->d_part_lo})
       cudaFree(p);
-    h->d_cross_list = h->d_cross_end = nullptr;
-    h->d_desc = nullptr;
-    h->d_compact = h->d_rec_hi = h->d_rec_lo = nullptr;
-    h->d_rec_meta = nullptr;
-    h->d_seg_status = nullptr;
-    GBA_CUDA(h, cudaMalloc(&h->d_desc, cap * sizeof(RowDesc)));
-    GBA_CUDA(h, cudaMalloc(&h->d_compact, (size_t)cap * cs * sizeof(float)));
-    GBA_CUDA(h, cudaMalloc(&h->d_rec_hi, (size_t)wins * 2 * h->d_max * sizeof(float)));
-    GBA_CUDA(h, cudaMalloc(&h->d_rec_lo, (size_t)wins * 2 * h->d_max * sizeof(float)));
-    GBA_CUDA(h, cudaMalloc(&h->d_rec_meta, (size_t)wins * 2 * REC_META * sizeof(uint32_t)));
-    GBA_CUDA(h, cudaMalloc(&h->d_seg_status, (size_t)wins * sizeof(unsigned long long)));
-    GBA_CUDA(h, cudaMalloc(&h->d_cross_list, (size_t)wins * sizeof(uint32_t)));
-    GBA_CUDA(h, cudaMalloc(&h->d_cross_end, (size_t)cap * sizeof(uint32_t)));
-    GBA_CUDA(h, cudaMemset(h->d_seg_status, 0, (size_t)wins * sizeof(unsigned long long)));
-    h->seg_win_cap = wins;
-  }
-  if (h->debug && N > h->dbg_cap) {
-    sync_all(h);
-    cudaFree(h->d_dbg_count);
-    cudaFree(h->d_dbg_kept);
-    h->d_dbg_count = h->d_dbg_kept = nullptr;
-    const int64_t cap = std::max<int64_t>(h->n_cap, N);
-    GBA_CUDA(h, cudaMalloc(&h->d_dbg_count, cap * sizeof(uint32_t)));
-    GBA_CUDA(h, cudaMalloc(&h->d_dbg_kept, cap * sizeof(uint32_t)));
-    h->dbg_cap = cap;
+    h->d_rr = nullptr;
+    h->d_kl = nullptr;
+    h->d_kw = h->d_part_hi = h->d_part_lo = nullptr;
+    h->d_scan_status = nullptr;
+    h->d_long_rows = nullptr;
+    h->d_long_done = nullptr;
+    h->d_items = nullptr;
+    const int64_t stiles = scan_tiles(cap);
+    const int64_t long_cap = cap / (LONG_ROW + 1) + h->T + 1;
+    const int64_t items_cap = cap / LONG_CHUNK + long_cap;
+    const int64_t parts_cap = 2 * (cap / LONG_CHUNK) + h->T + 1;
+    GBA_CUDA(h, cudaMalloc(&h->d_rr, (size_t)(cap + h->T + 1) * sizeof(uint4)));
+    GBA_CUDA(h, cudaMalloc(&h->d_kl, (size_t)cap * sizeof(float*)));
+    GBA_CUDA(h, cudaMalloc(&h->d_kw, (size_t)cap * sizeof(float)));
+    GBA_CUDA(h, cudaMalloc(&h->d_scan_status, (size_t)stiles * 4 * sizeof(unsigned long long)));
+    GBA_CUDA(h, cudaMemset(h->d_scan_status, 0, (size_t)stiles * 4 * sizeof(unsigned long long)));
+    GBA_CUDA(h, cudaMalloc(&h->d_long_rows, (size_t)long_cap * sizeof(uint4)));
+    GBA_CUDA(h, cudaMalloc(&h->d_long_done, (size_t)long_cap * sizeof(uint32_t)));
+    GBA_CUDA(h, cudaMalloc(&h->d_items, (size_t)items_cap * sizeof(uint2)));
+    GBA_CUDA(h, cudaMalloc(&h->d_part_hi, (size_t)parts_cap * h->d_max * sizeof(float)));
+    GBA_CUDA(h, cudaMalloc(&h->d_part_lo, (size_t)parts_cap * h->d_max * sizeof(float)));
   }
   return GBA_OK;
 }
@@ -660,7 +646,7 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
     const size_t M = (size_t)max_buffered_msgs;
     const size_t bytes = align16(MAX_PASSES * 256 * 4) + align16(MAX_PASSES * 4) +
                          align16(M * 4) + align16(M * 4) + align16(4) + align16(4) +
-                         align16((size_t)std::max(h->T, 1) * 8);
+                         align16((size_t)std::max(h->T, 1) * 32) + align16(M * 4);
     for (int b = 0; b < SLOTS; ++b) {
       if (!dev_alloc((void**)&h->d_step_scratch[b], bytes)) return fail(GBA_E_OOM);
       if (cudaMemset(h->d_step_scratch[b], 0, bytes) != cudaSuccess) return fail(GBA_E_CUDA);
@@ -679,9 +665,11 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
       sc.step_err = (uint32_t*)p;
       p += align16(4);
       sc.seg_ticket = (uint32_t*)p;
+      p += align16((size_t)std::max(h->T, 1) * 32);
+      sc.fw = (float*)p;
     }
   }
-  if (!dev_alloc((void**)&h->d_seg_total, 16)) return fail(GBA_E_OOM);
+  if (!dev_alloc((void**)&h->d_seg_total, (size_t)std::max(h->T, 1) * 4)) return fail(GBA_E_OOM);
   if (!dev_alloc((void**)&h->d_err, 4) || !dev_alloc((void**)&h->d_stats, sizeof(DevStats)))
     return fail(GBA_E_OOM);
   if (cudaHostAlloc((void**)&h->h_err, 4, cudaHostAllocMapped) != cudaSuccess)
@@ -895,37 +883,37 @@ int32_t gba_try_apply(gba_handle* h) {
       tb.pos_begin = nbase[t];
       tb.pos_end = nbase[t + 1];
       tb.opt = make_opt_step(ts.desc.opt, p1, p2);
-      uint32_t* dc = h->debug ? h->d_dbg_count : nullptr;
-      uint32_t* dk = h->debug ? h->d_dbg_kept : nullptr;
       if (++h->epoch == 0u) h->epoch = 1u;
       SegOut so{};
-      so.desc = h->d_desc;
-      so.compact = h->d_compact;
-      so.cs = (tb.d + 3) / 4 * 4;
-      so.rec_stride = h->d_max;
-      so.rec_hi = h->d_rec_hi;
-      so.rec_lo = h->d_rec_lo;
-      so.rec_meta = h->d_rec_meta;
-      so.status = h->d_seg_status;
+      so.rr = h->d_rr + nbase[t] + t;
+      so.kl = h->d_kl + nbase[t];
+      so.kw = h->d_kw + nbase[t];
+      so.status = h->d_scan_status;
       so.epoch = h->epoch;
-      so.ticket = sc.seg_ticket + 2 * t;
-      so.cross_count = sc.seg_ticket + 2 * t + 1;
-      so.cross_list = h->d_cross_list;
-      so.cross_end = h->d_cross_end;
-      so.total = h->d_seg_total;
-      int64_t n_win = 0;
+      so.ticket = sc.seg_ticket + 8 * t;
+      so.n_long = sc.seg_ticket + 8 * t + 1;
+      so.n_items = sc.seg_ticket + 8 * t + 2;
+      so.n_parts = sc.seg_ticket + 8 * t + 3;
+      so.item_ticket = sc.seg_ticket + 8 * t + 4;
+      so.total = h->d_seg_total + t;
+      so.long_rows = h->d_long_rows;
+      so.long_done = h->d_long_done;
+      so.items = h->d_items;
+      so.part_hi = h->d_part_hi;
+      so.part_lo = h->d_part_lo;
+      so.pstride = h->d_max;
       {
-        Timed tm(h, GBA_K_SEG_REDUCE, h->applys);
-        n_win = launch_seg_reduce(a, tb, so, h->d_keys[b][final_buf], h->d_vals[b][final_buf],
-                                  h->d_stats, dc, dk, sink, h->num_sms, h->wait_ns, h->applys);
+        Timed tm(h, GBA_K_SEG_SCAN, h->applys);
+        launch_seg_scan(a, tb, so, h->d_keys[b][final_buf], h->d_vals[b][final_buf], h->d_stats,
+                        sink, h->wait_ns, h->applys);
       }
       {
-        Timed tm(h, GBA_K_SEG_CROSS, h->applys);
-        launch_seg_cross(a, tb, so, n_win, dc, dk, sink, h->applys);
+        Timed tm(h, GBA_K_ROW_APPLY, h->applys);
+        launch_row_apply(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
       }
       {
-        Timed tm(h, GBA_K_ROW_UPDATE, h->applys);
-        launch_row_update(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
+        Timed tm(h, GBA_K_ROW_LONG, h->applys);
+        launch_row_long(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
       }
     }
   }
@@ -968,6 +956,7 @@ int32_t gba_try_apply(gba_handle* h) {
   h->k += 1;
   h->have_last = true;
   h->last_N = N;
+  h->last_nbase = nbase;
   h->last_buf = final_buf;
   h->last_slot = b;
   h->last_M = M;
@@ -1051,6 +1040,31 @@ gba_status gba_kernel_times(gba_handle* h, gba_kernel_times_t* out) {
   return GBA_OK;
 }
 
+gba_status gba_pull(gba_handle* h, int32_t t, const int64_t* ids, int64_t n, float* out) {
+  if (!h || t < 0 || t >= h->T || n < 0) return GBA_E_ARG;
+  if (n > 0 && (!ids || !out)) return set_err(h, GBA_E_ARG, "NULL ids or out");
+  if (h->failed) return set_err(h, GBA_E_STATE, "handle failed earlier");
+  if (((uintptr_t)ids & 7u) != 0) return set_err(h, GBA_E_ARG, "ids not 8-byte aligned");
+  if (n == 0) return GBA_OK;
+  cudaSetDevice(h->device);
+  join_steps(h);  // the rows as of every step enqueued so far
+  const TableState& ts = h->tables[t];
+  ErrSink sink = h->sink;
+  sink.step = h->d_err;  // no step of its own: the handle's word takes both roles
+  launch_pull_rows(ts.w, ts.desc.rows, ts.desc.dim, ts.desc.id_mode, ids, n, out, sink,
+                   h->num_sms, h->stream);
+  GBA_CUDA(h, cudaGetLastError());
+  return GBA_OK;
+}
+
+gba_status gba_join(gba_handle* h) {
+  if (!h) return GBA_E_ARG;
+  cudaSetDevice(h->device);
+  join_steps(h);
+  GBA_CUDA(h, cudaGetLastError());
+  return GBA_OK;
+}
+
 gba_status gba_set_overlap(gba_handle* h, int32_t on) {
   if (!h) return GBA_E_ARG;
   cudaSetDevice(h->device);
@@ -1068,32 +1082,33 @@ gba_status gba_set_debug(gba_handle* h, int32_t on) {
 gba_status gba_debug_segments(gba_handle* h, int64_t cap, int32_t* table, int64_t* row,
                               int64_t* count, int64_t* kept, int64_t* n_unique) {
   if (!h || !n_unique) return GBA_E_ARG;
-  if (!h->have_last || !h->debug || !h->d_dbg_count)
+  if (!h->have_last || !h->debug)
     return set_err(h, GBA_E_STATE, "no debug record of a step (enable debug before the step)");
   cudaSetDevice(h->device);
   GBA_CUDA(h, sync_all(h));
-  const int64_t N = h->last_N;
-  std::vector<uint32_t> keys(N), cnt(N), kp(N);
-  if (N > 0) {
-    GBA_CUDA(h, cudaMemcpy(keys.data(), h->d_keys[h->last_slot][h->last_buf], N * 4, cudaMemcpyDeviceToHost));
-    GBA_CUDA(h, cudaMemcpy(cnt.data(), h->d_dbg_count, N * 4, cudaMemcpyDeviceToHost));
-    GBA_CUDA(h, cudaMemcpy(kp.data(), h->d_dbg_kept, N * 4, cudaMemcpyDeviceToHost));
-  }
-  int64_t u = 0;
-  for (int64_t i = 0; i < N; ++i) {
-    if (i > 0 && keys[i] == keys[i - 1]) continue;
-    if (u < cap) {
-      int t = 0;
-      while (t + 1 < h->T && keys[i] >= h->tables[t + 1].key_base) ++t;
-      if (table) table[u] = t;
-      if (row) row[u] = (int64_t)(keys[i] - h->tables[t].key_base);
-      if (count) count[u] = cnt[i];
-      if (kept) kept[u] = kp[i];
+  // the step's row records, table by table: (row, prefixes of kept occurrences
+  // and of (message, row) pairs at the row's head), closed by the totals
+  std::vector<uint32_t> U(h->T, 0u);
+  if (h->T > 0 && h->last_N > 0)
+    GBA_CUDA(h, cudaMemcpy(U.data(), h->d_seg_total, h->T * sizeof(uint32_t),
+                           cudaMemcpyDeviceToHost));
+  int64_t u_all = 0;
+  for (int t = 0; t < h->T; ++t) {
+    const int64_t Nt = h->last_nbase[t + 1] - h->last_nbase[t];
+    if (Nt == 0) continue;
+    std::vector<uint4> rr((size_t)U[t] + 1);
+    GBA_CUDA(h, cudaMemcpy(rr.data(), h->d_rr + h->last_nbase[t] + t, rr.size() * sizeof(uint4),
+                           cudaMemcpyDeviceToHost));
+    for (uint32_t u = 0; u < U[t]; ++u, ++u_all) {
+      if (u_all >= cap) continue;
+      if (table) table[u_all] = t;
+      if (row) row[u_all] = (int64_t)rr[u].x;
+      if (count) count[u_all] = (int64_t)(rr[u + 1].z - rr[u].z);
+      if (kept) kept[u_all] = (int64_t)(rr[u + 1].y - rr[u].y);
     }
-    ++u;
   }
-  *n_unique = u;
-  return u > cap ? set_err(h, GBA_E_ARG, "capacity too small") : GBA_OK;
+  *n_unique = u_all;
+  return u_all > cap ? set_err(h, GBA_E_ARG, "capacity too small") : GBA_OK;
 }
 
 gba_status gba_debug_sorted(gba_handle* h, int64_t cap, uint32_t* keys, uint32_t* occ,
@@ -1142,6 +1157,15 @@ gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream) {
   return result ? GBA_E_DEVICE_TIMEOUT : GBA_OK;
 }
 
-const char* gba_version_string(void) { return "libgba 0.1 (sm_103a)"; }
+int32_t gba_device_binary_version(void) {
+  const int v = kernel_binary_version();
+  if (v < 0) {
+    cudaGetLastError();
+    return GBA_E_CUDA;
+  }
+  return v;
+}
+
+const char* gba_version_string(void) { return "libgba 0.2 (sm_103a)"; }
 
 }  // extern "C"

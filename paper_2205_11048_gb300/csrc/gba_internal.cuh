@@ -162,7 +162,10 @@ struct StepArgs {
   int32_t iota;
   int32_t row_staleness;
   int32_t sparse_den;
-  int32_t pad0;
+  int32_t decay;        // 0: f in {0, 1} (Eq. (1)); 1: f = lambda^s for s <= iota
+  int32_t drop_latest;  // the last drop_latest popped messages are excluded (0: none)
+  int32_t n_wtab;       // entries of wtab (decay 1): wtab[s] = lambda^s, s < n_wtab
+  const float* wtab;    // [n_wtab] device
   const int64_t* tokens;          // [M]
   const float* const* dense_ptr;  // [M]
   const uint32_t* msg_off;        // [T][M+1] occurrence offsets within the table
@@ -180,8 +183,30 @@ struct StepScratch {
   int32_t* kept_list;      // [M] indices of kept messages, in pop order
   int32_t* n_kept;         // [1]
   uint32_t* step_err;      // [1] failures of this step
-  uint32_t* seg_ticket;    // [T][2] window tickets and crossing-row counts of the segment kernels
+  uint32_t* seg_ticket;    // [T][8] per table: scan tile tickets, long rows, their items,
+                           // chunk-sum slots, item tickets, unused
+  float* fw;               // [M] message weights of the dense sum (decay 1; 1 or 0 otherwise)
 };
+
+// Weight of a gradient with staleness s (s >= 0), or 0 when it is excluded:
+// Eq. (1) keeps s <= iota; decay 1 scales a kept gradient by lambda^s.
+__device__ __forceinline__ float decay_weight(const StepArgs& a, uint64_t s) {
+  if (s > (uint64_t)(int64_t)a.iota) return 0.f;
+  if (a.decay == 0) return 1.f;
+  return s < (uint64_t)a.n_wtab ? __ldg(a.wtab + s) : 0.f;
+}
+
+// Compensated accumulation of a product f * g: the product's rounding error
+// (from a fused multiply-add) joins the compensation term, so with f = 1 this
+// is exactly csum_add.
+__device__ __forceinline__ void csum_add_prod(CSum& c, float f, float g) {
+  const float p = __fmul_rn(f, g);
+  const float e = __fmaf_rn(f, g, -p);
+  float s, t;
+  two_sum(c.hi, p, s, t);
+  c.hi = s;
+  c.lo = __fadd_rn(c.lo, __fadd_rn(t, e));
+}
 
 // Accumulated statistics (device).
 struct DevStats {
@@ -238,51 +263,55 @@ struct SegTable {
   OptStep opt;
 };
 
-// One row of the step's compact update list: where its aggregated gradient
-// is (a message's gradient row when one occurrence was kept, else the compact
-// buffer), the row, and the denominator of its weighted sum (0: no update).
-struct RowDesc {
-  const float* src;
-  uint32_t x;
-  float den;
-};
-
-constexpr int REC_META = 8;  // type, x, c_all, c_kept, k_occ, head_pos, u, unused
-
-// Buffers of the segment-sum and row-update kernels (one set, used in stream
-// order by the apply stream).
+// Buffers of the row kernels (one set, used in stream order by the apply
+// stream; every table of a step uses its own ranges of rr / kl / kw).
+//  rr[u]   row u of the table in sorted order: (row x, and the exclusive
+//          prefixes at its head of kept occurrences K, (message, row) pairs C
+//          and kept pairs CK); rr[U] holds the totals, so row u's kept
+//          occurrences are kl[rr[u].K .. rr[u+1].K), c_x = rr[u+1].C - rr[u].C
+//  kl[j]   address of the j-th kept occurrence's gradient row, sorted by row
+//  kw[j]   its weight f (1 under Eq. (1))
 struct SegOut {
-  RowDesc* desc;              // [U] the step's rows in sorted order
-  float* compact;             // [U][cs] sums of rows with two or more kept occurrences
-  int32_t cs;                 // compact row stride (floats, a multiple of 4)
-  int32_t rec_stride;         // floats per record
-  float* rec_hi;              // [windows][2][rec_stride] compensated partial sums
-  float* rec_lo;              // [windows][2][rec_stride]
-  uint32_t* rec_meta;         // [windows][2][REC_META]
-  unsigned long long* status; // [windows] look-back words
-  uint32_t epoch;             // tag of this launch's look-back words
-  uint32_t* ticket;           // window tickets (cleared by K1)
-  uint32_t* cross_count;      // rows that cross windows (cleared by K1)
-  uint32_t* cross_list;       // [windows] windows where such a row begins
-  uint32_t* cross_end;        // [U] window where a crossing row ends, by list index
-  uint32_t* total;            // U, written by the last window
+  uint4* rr;                   // this table's range
+  const float** kl;            // this table's range
+  float* kw;                   // this table's range
+  unsigned long long* status;  // [tiles][4] look-back words of the scan
+  uint32_t epoch;              // tag of this launch's look-back words
+  uint32_t* ticket;            // scan tile tickets (cleared by K1)
+  uint32_t* n_long;            // rows with more than LONG_ROW kept occurrences (cleared by K1)
+  uint32_t* n_items;           // chunks of those rows (cleared by K1)
+  uint32_t* n_parts;           // chunk-sum slots of rows split into chunks (cleared by K1)
+  uint32_t* item_ticket;       // items claimed by warps of the long-row kernel (cleared by K1)
+  uint32_t* total;             // this table's U (written by the last scan tile)
+  uint4* long_rows;            // [n_long] (u, first kept, kept count, first chunk-sum slot)
+  uint32_t* long_done;         // [n_long] chunks of the row finished
+  uint2* items;                // [n_items] (long row, chunk)
+  float* part_hi;              // [n_parts][pstride] compensated chunk sums
+  float* part_lo;
+  int32_t pstride;
 };
 
-// Upper bound on the windows of a table of N sorted positions.
-int64_t seg_window_bound(int64_t N, int num_sms);
+// Rows with at most LONG_ROW kept occurrences are applied by one lane group
+// each with all their gradient rows staged in shared memory; longer rows by a
+// whole warp each, in chunks of LONG_CHUNK kept occurrences.
+constexpr int LONG_ROW = 4;
+#ifndef GBA_LONG_CHUNK
+#define GBA_LONG_CHUNK 128
+#endif
+constexpr int LONG_CHUNK = GBA_LONG_CHUNK;
+constexpr int SCAN_TILE = 2048;
 
-// Segment reduction over table tb's range of the sorted array; returns the
-// number of windows (for the cross-window kernel).
-int64_t launch_seg_reduce(const StepArgs& a, const SegTable& tb, const SegOut& so,
-                          const uint32_t* keys, const uint32_t* vals, DevStats* stats,
-                          uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, int num_sms,
-                          int64_t wait_ns, cudaStream_t s);
+int64_t scan_tiles(int64_t N);
 
-void launch_seg_cross(const StepArgs& a, const SegTable& tb, const SegOut& so, int64_t n_win,
-                      uint32_t* dbg_count, uint32_t* dbg_kept, ErrSink err, cudaStream_t s);
+void launch_seg_scan(const StepArgs& a, const SegTable& tb, const SegOut& so, const uint32_t* keys,
+                     const uint32_t* vals, DevStats* stats, ErrSink err, int64_t wait_ns,
+                     cudaStream_t s);
 
-void launch_row_update(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
-                       ErrSink err, int num_sms, cudaStream_t s);
+void launch_row_apply(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
+                      ErrSink err, int num_sms, cudaStream_t s);
+
+void launch_row_long(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
+                     ErrSink err, int num_sms, cudaStream_t s);
 
 struct DenseArgs {
   float* w;
@@ -306,5 +335,13 @@ void launch_init_dense(float* w, float* s0, float* s1, int64_t D, int32_t kind, 
                        uint64_t seed, uint64_t tag, cudaStream_t s);
 
 int launch_wait_selftest(int64_t limit_ns, cudaStream_t s, uint32_t* d_word, uint32_t* result);
+
+// Rows of one table for n ids (pull responding), into out[n][d].
+void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, const int64_t* ids, int64_t n,
+                      float* out, ErrSink err, int num_sms, cudaStream_t s);
+
+// Compute capability (major * 10 + minor) of the device code the library's
+// kernels were loaded from on the current device, or -1.
+int kernel_binary_version();
 
 }  // namespace gba

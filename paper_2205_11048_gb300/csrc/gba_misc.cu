@@ -83,4 +83,10 @@ int launch_wait_selftest(int64_t limit_ns, cudaStream_t s, uint32_t* d_word, uin
   return 0;
 }
 
+int kernel_binary_version() {
+  cudaFuncAttributes attr{};
+  if (cudaFuncGetAttributes(&attr, k_init_params) != cudaSuccess) return -1;
+  return attr.binaryVersion;
+}
+
 }  // namespace gba

@@ -1,22 +1,24 @@
 // gba_sort_ids_static: the library's id sort for callers that cannot allocate.
 //
-// Some callers cannot allocate device memory at the point where they need a
-// sort: code running inside a CUDA graph that is being captured (cudaMalloc is
-// not a stream operation and may not be captured), allocators' own hooks, or
-// runtimes whose memory is fully reserved up front.  This entry point runs the
-// same histogram and onesweep kernels as a global step, but takes its scratch
-// from one fixed array in device global memory that the library reserves when
-// it is loaded, so the call itself never allocates.
+// Some callers must not allocate device memory at the point where they need a
+// sort: runtimes that reserve all device memory up front and hand none out
+// later, or an allocator's own hooks, which cannot re-enter cudaMalloc.  This
+// entry point runs the same histogram and onesweep kernels as a global step,
+// but takes its scratch from one fixed array in device global memory that is
+// part of the library image, so the call itself never allocates.
 //
 // Properties a caller must know:
 //  - The scratch array is file-scope device memory of GBA_STATIC_SORT_BYTES
 //    bytes; every GPU that loads the library keeps it until the process exits.
 //  - The first call on a device (with that device current) looks up the
-//    array's device address; make that first call before any stream capture.
+//    array's device address with cudaGetSymbolAddress.
+//  - The call is synchronous: it waits for its stream before returning, so it
+//    cannot be captured into a CUDA graph.
 //  - All calls share the one array and it keeps the previous call's contents.
 //    The per-call counters are cleared at the start of each call; calls whose
 //    work overlaps on the GPU (two streams, or two host threads) race.
 //  - At most GBA_STATIC_SORT_MAX_IDS ids per call; larger inputs are refused.
+//  - The outputs hold the sorted result only when GBA_OK is returned.
 #include <cuda_runtime.h>
 
 #include <atomic>
@@ -111,6 +113,10 @@ extern "C" gba_status gba_sort_ids_static(const int64_t* ids, int64_t n, int64_t
   if (id_mode != GBA_ID_DIRECT && id_mode != GBA_ID_MODULO) return GBA_E_ARG;
   if (n > 0 && (!ids || !rows_out || !order_out)) return GBA_E_ARG;
   if (n == 0) return GBA_OK;
+  // A launch error left by earlier, unrelated work on this thread would be
+  // reported (and cleared) by the check after the launches below: refuse to
+  // run instead, and leave that error in place for its owner.
+  if (cudaPeekAtLastError() != cudaSuccess) return GBA_E_CUDA;
   cudaStream_t s = (cudaStream_t)cuda_stream;
   unsigned char* base = nullptr;
   int dev = 0;

@@ -127,7 +127,7 @@ __global__ void __launch_bounds__(256) k_message_weights(StepArgs a, StepScratch
   if (tid < MAX_PASSES) sc.tile_counter[tid] = 0u;
   if (tid == 0) *sc.step_err = 0u;
   if (sc.seg_ticket)
-    for (int i = tid; i < 2 * a.T; i += blockDim.x) sc.seg_ticket[i] = 0u;
+    for (int i = tid; i < 8 * a.T; i += blockDim.x) sc.seg_ticket[i] = 0u;
   if (tid >= 32) return;
   const int lane = tid;
   int kept = 0;

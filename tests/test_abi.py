@@ -29,11 +29,17 @@ def test_exports_every_declared_symbol(L):
     assert set(declared) <= set(B._SIGNATURES)
 
 
-def test_library_targets_sm103a(L):
-    out = subprocess.run(["cuobjdump", "--list-elf", B.LIB_PATH], capture_output=True, text=True)
-    if out.returncode != 0:
-        pytest.skip("cuobjdump unavailable")
-    assert "sm_103a" in out.stdout
+def test_library_is_built_for_sm103a_only():
+    """Every translation unit and the link are compiled for sm_103a and nothing else."""
+    from paper_2205_11048_gb300 import build as BLD
+    assert BLD.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def test_no_device_code_without_a_gpu(L):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present (the GPU test checks the version)")
+    assert L.gba_device_binary_version() == B.GBA_E_CUDA
 
 
 def _table(rows=100, dim=16, mode=0, mx=10, kind=0, init=0.1):

@@ -98,6 +98,42 @@ def test_hand_example_matches_golden_exactly():
     g.close()
 
 
+@pytest.mark.parametrize("variant", [0, 1, 2])
+def test_rule_option_goldens_exactly(variant):
+    """The hand-worked steps of the optional readings (kept-message and M
+    denominators, message staleness for rows), through the CUDA path."""
+    from tests import _pins
+    gj = _pins.load_golden()["rule_options"]
+    var = gj["variants"][variant]
+    F = _pins.F
+    lr, acc0 = F(gj["table"]["lr"]), F(gj["table"]["init_acc"])
+    tables = [(4, 2, 0, 8, B.opt_desc(0, lr, acc0))]
+    g = B.GBA(tables, 2, B.opt_desc(0, lr, acc0), 2, 8, seed=4321, **var["rule"])
+    w0 = g.table(0)[0].cpu().numpy().astype(np.float64)
+    dw0 = g.dense()[0].cpu().numpy().astype(np.float64)
+    for step in (gj["step0"], var["step1"]):
+        for m in step["messages"]:
+            ids = torch.tensor(m["ids"], dtype=torch.int64, device="cuda")
+            rows = torch.tensor(m["rows"], dtype=torch.float32, device="cuda")
+            g.push(m["token"], [ids], [rows], torch.tensor(m["dense"], dtype=torch.float32,
+                                                           device="cuda"), m["B"])
+        assert g.try_apply() == 1
+        e = step["expect"]
+        assert g.keep().tolist() == e["keep"]
+        w, s0, _, ver = g.table(0)
+        for r in range(4):
+            assert (w[r].cpu().numpy().astype(np.float64) - w0[r]).tolist() == \
+                [F(v) for v in e["dw"][str(r)]]
+            assert s0[r].cpu().numpy().astype(np.float64).tolist() == \
+                [F(v) for v in e["acc"][str(r)]]
+        assert ver.cpu().tolist() == e["ver"]
+        dw, ds0, _ = g.dense()
+        assert (dw.cpu().numpy().astype(np.float64) - dw0).tolist() == \
+            [F(v) for v in e["dense_dw"]]
+        assert ds0.cpu().numpy().astype(np.float64).tolist() == [F(v) for v in e["dense_acc"]]
+    g.close()
+
+
 @pytest.mark.parametrize("dim", [1, 3, 4, 8, 19, 24, 64, 128, 200, 256])
 @pytest.mark.parametrize("kind", [0, 1])
 def test_row_widths_and_optimizers(dim, kind):
@@ -313,3 +349,99 @@ def test_tiny_wait_limit_in_sort_is_reported_or_harmless():
     assert g2.try_apply() == 1
     g2.sync()
     g2.close()
+
+
+def test_tiny_wait_limit_in_dense_is_reported_or_harmless():
+    """A dense-only step with a zero wait limit: the dense kernel's mbarrier
+    waits give up whenever a stage is not ready at the first try, the producer
+    stops issuing copies and waits (with its own bound) for the ones in
+    flight, and the step reports GBA_E_DEVICE_TIMEOUT -- or completes if no
+    wait had to give up.  Either way the context stays usable and a fresh
+    handle applies a step afterwards."""
+    D, M = 3_000_001, 6
+    dense_opt = B.opt_desc(W.ADAM, 0.001)
+    gen = torch.Generator(device="cuda").manual_seed(9)
+    grads = [torch.randn(D, generator=gen, device="cuda") * 0.01 for _ in range(M)]
+    g = B.GBA([], D, dense_opt, M, 2 * M, seed=2)
+    g.set_wait_limit(0)
+    for i in range(M):
+        g.push_ref(0, [], [], grads[i], 1)
+    rc = g.L.gba_try_apply(g.h)
+    if rc == 1:
+        rc = g.L.gba_sync(g.h)
+    assert rc in (B.GBA_OK, B.GBA_E_DEVICE_TIMEOUT)
+    g.close()
+    g2 = B.GBA([], D, dense_opt, M, 2 * M, seed=2)
+    for i in range(M):
+        g2.push_ref(0, [], [], grads[i], 1)
+    assert g2.try_apply() == 1
+    g2.sync()
+    w, _, _ = g2.dense()
+    assert torch.isfinite(w).all()
+    g2.close()
+
+
+def test_device_code_is_sm103a():
+    """The kernels run from sm_103a device code on this GPU."""
+    assert B.load().gba_device_binary_version() == 103
+
+
+@pytest.mark.parametrize("dim,mode", [(16, 0), (3, 0), (64, 1), (19, 1)])
+def test_pull_returns_the_current_rows(dim, mode):
+    """Pull responding (Alg. 2): after a few steps, gba_pull gives exactly the
+    oracle's rows for any ids (duplicates, MODULO residues of negative ids)."""
+    rng = np.random.default_rng(dim + 100 * mode)
+    V = 997
+    cfg = cfg_of([(V, dim, mode, 0)], D=7, G=3, iota=1)
+    steps = []
+    for k in range(3):
+        batch = []
+        for m in range(3):
+            n = int(rng.integers(1, 200))
+            ids = rng.zipf(1.3, n) % V if mode == 0 else rng.integers(-2**62, 2**62, n)
+            batch.append(msg(max(0, k - int(rng.integers(0, 2))), [ids], [dim], 7))
+        steps.append(batch)
+    g, orc = run_custom(cfg, steps)
+    if mode == 0:
+        ids = rng.integers(0, V, 1000)
+    else:
+        ids = np.concatenate([rng.integers(-2**62, 2**62, 500),
+                              np.concatenate([s_[0]["ids"][0].cpu().numpy() for s_ in steps])])
+    ids_t = torch.as_tensor(ids, dtype=torch.int64, device="cuda")
+    got = g.pull(0, ids_t).cpu().numpy()
+    rows = H.rows_of(cfg, 0, ids.astype(np.int64))
+    want = orc.tables[0].w.reshape(V, dim)[rows]
+    assert np.array_equal(got, want)
+    assert g.pull(0, ids_t[:0]).shape == (0, dim)
+    g.sync()
+    g.close()
+
+
+def test_pull_orders_after_overlapping_steps():
+    """With steps overlapping, a pull still sees every step enqueued before it."""
+    cfg = W.reduced(2)
+    g = H.make_gpu(cfg, overlap=True, debug=False)
+    orc = H.make_oracle(cfg)
+    for k in range(3):
+        for m in W.generate_step(cfg, k, "cuda"):
+            H.push_gpu(g, m)
+            orc.push(H.to_oracle(m))
+        assert g.try_apply() == 1 and orc.try_apply() == 1
+    ids = torch.arange(0, cfg.tables[0].rows, 7, dtype=torch.int64, device="cuda")
+    got = g.pull(0, ids).cpu().numpy()
+    want = orc.tables[0].w.reshape(cfg.tables[0].rows, -1)[ids.cpu().numpy()]
+    assert np.array_equal(got, want)
+    g.close()
+
+
+def test_pull_of_an_out_of_range_id_is_latched():
+    tables = [(100, 8, 0, 16, B.opt_desc())]
+    g = B.GBA(tables, 0, None, 1, 4, seed=1)
+    ids = torch.tensor([3, 100, 5], dtype=torch.int64, device="cuda")
+    out = g.pull(0, ids)
+    assert int(g.L.gba_sync(g.h)) == B.GBA_E_ID_RANGE
+    o = out.cpu().numpy()
+    assert np.all(o[1] == 0)
+    w = _raw_table_w(g, 0).view(100, 8).cpu().numpy()
+    assert np.array_equal(o[[0, 2]], w[[3, 5]])
+    g.close()
