@@ -75,6 +75,11 @@ typedef struct {
   int32_t iota;                /* tolerance threshold of Eq. (1); INT32_MAX = keep all */
   int32_t row_staleness;       /* 0: tag of the ID vs token, 1: k vs token */
   int32_t sparse_denominator;  /* 0: messages that contain the ID, 1: kept ones, 2: M */
+  int32_t decay;               /* 0: Eq. (1) as printed (weight 1 or 0);
+                                  1: a kept gradient of staleness s weighs lambda^s */
+  float lambda;                /* decay 1 only: 0 < lambda <= 1 */
+  int32_t drop_latest;         /* Hop-BW backup workers: the last drop_latest popped
+                                  gradients of a step are ignored (0: none) */
 } gbao_rule;
 
 /* Counters of one step (Table 3 reports dropped batches and staleness). */
@@ -209,6 +214,21 @@ static int64_t staleness(int64_t ref, int64_t token) {
   return s < 0 ? 0 : s;
 }
 
+/* The weight of a gradient with staleness s from the m-th popped message of
+ * M.  Eq. (1): 0 beyond iota, else 1.  Sec. 4.1 leaves room for other decay
+ * strategies; decay 1 weighs a kept gradient by lambda^s (s successive
+ * multiplications in double, rounded once to float).  Sec. 5.1's Hop-BW
+ * ignores the gradients of the slowest workers: with drop_latest = b3 the
+ * last b3 popped messages weigh 0. */
+static float decay_weight(const gbao_rule* rule, int64_t s, int32_t m, int32_t M) {
+  if (s > (int64_t)rule->iota) return 0.0f;
+  if (m >= M - rule->drop_latest) return 0.0f;
+  if (rule->decay == 0) return 1.0f;
+  double p = 1.0;
+  for (int64_t i = 0; i < s; ++i) p = p * (double)rule->lambda;
+  return (float)p;
+}
+
 /*
  * One global step k over the M popped messages.
  *
@@ -231,15 +251,16 @@ int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens
   gbao_stats st;
   memset(&st, 0, sizeof st);
 
-  /* Eq. (1): f(tau(m,k), k) = 0 if k - tau > iota, else 1. */
-  int32_t* f = (int32_t*)malloc(sizeof(int32_t) * (size_t)(M > 0 ? M : 1));
+  /* Eq. (1): f(tau(m,k), k) = 0 if k - tau > iota, else 1 (or the weight of
+   * the chosen decay strategy). */
+  float* f = (float*)malloc(sizeof(float) * (size_t)(M > 0 ? M : 1));
   for (int32_t m = 0; m < M; ++m) {
     int64_t s = staleness(k, tokens[m]);
-    f[m] = (s <= (int64_t)rule->iota) ? 1 : 0;
-    if (f[m]) st.msgs_kept++; else st.msgs_dropped++;
+    f[m] = decay_weight(rule, s, m, M);
+    if (f[m] > 0.0f) st.msgs_kept++; else st.msgs_dropped++;
     st.dense_stale_sum += s;
     if (s > st.dense_stale_max) st.dense_stale_max = s;
-    if (keep_msg_out) keep_msg_out[m] = f[m];
+    if (keep_msg_out) keep_msg_out[m] = f[m] > 0.0f ? 1 : 0;
   }
 
   /* Adam bias corrections use the global step count t = k + 1. */
@@ -258,7 +279,7 @@ int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens
       int64_t e = dense->track[r];
       double S = 0.0;
       for (int32_t m = 0; m < M; ++m)
-        if (f[m]) S += (double)dense_grads[m][e];
+        if (f[m] > 0.0f) S += (double)f[m] * (double)dense_grads[m][e];
       float gsum = (float)S;
       float g = gsum / (float)M;
       apply_opt(&dense->opt, &dense->w[r], &dense->s0[r],
@@ -298,7 +319,8 @@ int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens
         st.occurrences++;
         int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k;
         int64_t s = staleness(ref, tokens[m]);
-        int keep = (s <= (int64_t)rule->iota);
+        float fo = decay_weight(rule, s, m, M);
+        int keep = fo > 0.0f;
         if (last_m[r] != m) {   /* first time row x is met in message m */
           last_m[r] = m;
           cnt[r]++;
@@ -309,7 +331,7 @@ int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens
         }
         if (keep) {
           kept_occ[r]++;
-          for (int32_t j = 0; j < d; ++j) S[r * d + j] += (double)gm[i * d + j];
+          for (int32_t j = 0; j < d; ++j) S[r * d + j] += (double)fo * (double)gm[i * d + j];
         }
       }
     }

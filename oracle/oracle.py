@@ -62,7 +62,8 @@ class _Dense(ctypes.Structure):
 
 class _Rule(ctypes.Structure):
     _fields_ = [("iota", ctypes.c_int32), ("row_staleness", ctypes.c_int32),
-                ("sparse_denominator", ctypes.c_int32)]
+                ("sparse_denominator", ctypes.c_int32), ("decay", ctypes.c_int32),
+                ("lambda_", ctypes.c_float), ("drop_latest", ctypes.c_int32)]
 
 
 class Stats(ctypes.Structure):
@@ -214,12 +215,14 @@ class OracleGBA:
 
     def __init__(self, tables, dense_size: int, dense_opt: OptSpec, global_batch: int,
                  iota: int = INT32_MAX, row_staleness: int = 0, sparse_denominator: int = 0,
-                 seed: int = 0, track_rows=None, track_dense=None, library=None):
+                 seed: int = 0, track_rows=None, track_dense=None, library=None, decay: int = 0,
+                 lam: float = 1.0, drop_latest: int = 0):
         self.L = library if library is not None else lib()
         self.specs = list(tables)
         self.D = int(dense_size)
         self.G = int(global_batch)
-        self.rule = _Rule(int(iota), int(row_staleness), int(sparse_denominator))
+        self.rule = _Rule(int(iota), int(row_staleness), int(sparse_denominator), int(decay),
+                          float(lam), int(drop_latest))
         self.k = 0
         self.fifo: list[Message] = []
         self.tables = []

@@ -112,6 +112,61 @@ def pin_hand_rule_options(L):
             _check_hand_step(orc, tb, step["expect"], w0, dw0)
 
 
+def pin_hand_decay_variants(L):
+    """Hand-worked steps of geometric decay (lambda^s) and of Hop-BW's ignored
+    latest gradients, exact in float32."""
+    g = load_golden()["decay_variants"]
+    for name in ("geometric", "hop_bw"):
+        var = g[name]
+        tb = O.TableSpec(g["table"]["rows"], g["table"]["dim"],
+                         O.OptSpec(O.ADAGRAD, F(g["table"]["lr"]), F(g["table"]["init_acc"])))
+        dopt = O.OptSpec(O.ADAGRAD, F(g["dense"]["lr"]), F(g["dense"]["init_acc"]))
+        orc = O.OracleGBA([tb], g["dense"]["D"], dopt, var["global_batch"], seed=4321, library=L,
+                          **var["rule"])
+        w0 = orc.tables[0].w.astype(np.float64).reshape(tb.rows, tb.dim).copy()
+        dw0 = orc.dense.w.astype(np.float64).copy()
+        for step in var["steps"]:
+            assert orc.pull_version() == step["k"]
+            for m in step["messages"]:
+                orc.push(_msg(m))
+            assert orc.try_apply() == 1
+            _check_hand_step(orc, tb, step["expect"], w0, dw0)
+
+
+def pin_decay_special_cases(L, seed=31):
+    """lambda = 1 is Eq. (1) and drop_latest = 0 ignores nothing: both give the
+    default rule's state bit for bit; drop_latest = M keeps no gradient, so
+    only the dense optimizer moves (with a zero gradient)."""
+    rng = np.random.default_rng(seed)
+    V, d, D, M = 11, 3, 7, 4
+    batches = [random_messages(rng, M, V, d, D, 0, 6, tokens=[max(0, s - int(t)) for t in
+                                                           rng.integers(0, 4, M)])
+               for s in range(4)]
+    def run(**rule):
+        tb = O.TableSpec(V, d, O.OptSpec(O.ADAM, 0.003))
+        orc = O.OracleGBA([tb], D, O.OptSpec(O.ADAM, 0.001), M, iota=2, seed=9, library=L, **rule)
+        for b in batches:
+            for m in b:
+                orc.push(m)
+            assert orc.try_apply() == 1
+        return orc
+    base = run()
+    for rule in (dict(decay=1, lam=1.0), dict(drop_latest=0)):
+        o = run(**rule)
+        assert np.array_equal(o.tables[0].w, base.tables[0].w), rule
+        assert np.array_equal(o.tables[0].ver, base.tables[0].ver), rule
+        assert np.array_equal(o.dense.w, base.dense.w), rule
+    none = run(drop_latest=M)
+    assert np.all(none.tables[0].ver == 0)
+    # with a zero gradient Adam's first step moves nothing: m = v = 0
+    tb = O.TableSpec(V, d, O.OptSpec(O.ADAM, 0.003))
+    fresh = O.OracleGBA([tb], D, O.OptSpec(O.ADAM, 0.001), M, iota=2, seed=9, library=L)
+    assert np.array_equal(none.dense.w, fresh.dense.w) and np.all(none.dense.s1 == 0)
+    # geometric weights fall with staleness: lambda^s for the kept dense gradients
+    o = run(decay=1, lam=0.5)
+    assert not np.array_equal(o.dense.w, base.dense.w)
+
+
 def pin_hand_adam(L):
     """One textbook Adam step with dyadic hyper-parameters."""
     g = load_golden()["adam"]
@@ -410,8 +465,9 @@ def pin_brute_force(L, seed=21):
         assert orc.dense.s0.tolist() == [float(v) for v in DS0]
 
 
-ALL_PINS = [pin_hand_adagrad, pin_hand_rule_options, pin_hand_adam, pin_sync_closed_form,
-            pin_decay_boundary, pin_fifo_prefix, pin_order_invariance, pin_brute_force]
+ALL_PINS = [pin_hand_adagrad, pin_hand_rule_options, pin_hand_decay_variants,
+            pin_decay_special_cases, pin_hand_adam, pin_sync_closed_form, pin_decay_boundary,
+            pin_fifo_prefix, pin_order_invariance, pin_brute_force]
 
 
 def pin_init_published(L):

@@ -13,9 +13,8 @@ SRC = os.path.join(os.path.dirname(O.__file__), "gba_oracle.c")
 
 # (name, original text, planted text, occurrence index to replace)
 MUTATIONS = [
-    ("dense-boundary-strict", "f[m] = (s <= (int64_t)rule->iota)", "f[m] = (s < (int64_t)rule->iota)", 0),
-    ("row-boundary-strict", "int keep = (s <= (int64_t)rule->iota);",
-     "int keep = (s < (int64_t)rule->iota);", 0),
+    ("decay-boundary-strict", "if (s > (int64_t)rule->iota) return 0.0f;",
+     "if (s >= (int64_t)rule->iota) return 0.0f;", 0),
     ("dense-divides-by-kept", "float g = gsum / (float)M;",
      "float g = gsum / (float)(st.msgs_kept > 0 ? st.msgs_kept : 1);", 0),
     ("row-divides-by-kept-messages", "int64_t denom = cnt[r];", "int64_t denom = cnt_kept[r];", 0),
@@ -25,13 +24,13 @@ MUTATIONS = [
      "int64_t ref = tokens[m];", 0),
     ("adagrad-sign", "*w = *w - step / den;", "*w = *w + step / den;", 0),
     ("adagrad-old-accumulator", "float den = sqrtf(an);", "float den = sqrtf(*a);", 0),
-    ("row-transposed", "S[r * d + j] += (double)gm[i * d + j];",
-     "S[r * d + j] += (double)gm[j * nm + i];", 0),
+    ("row-transposed", "S[r * d + j] += (double)fo * (double)gm[i * d + j];",
+     "S[r * d + j] += (double)fo * (double)gm[j * nm + i];", 0),
     ("no-skip-of-dropped-rows", "if (kept_occ[r] == 0) continue;", "if (kept_occ[r] < 0) continue;", 0),
     ("adam-step-count", "int64_t t_step = k + 1;", "int64_t t_step = k + 2;", 0),
     ("counts-occurrences", "if (last_m[r] != m) {", "if (1) {", 0),
     ("adam-moment-order", "float mn = o->beta1 * *m + c1 * g;", "float mn = c1 * *m + o->beta1 * g;", 0),
-    ("dense-drop-ignored", "if (f[m]) S += (double)dense_grads[m][e];",
+    ("dense-drop-ignored", "if (f[m] > 0.0f) S += (double)f[m] * (double)dense_grads[m][e];",
      "S += (double)dense_grads[m][e];", 0),
     ("init-scale", "return (float)top * 0x1p-27f;", "return (float)top * 0x1p-26f;", 0),
     ("fifo-overshoot", "if (acc >= G) return i + 1;", "if (acc > G) return i + 1;", 0),
@@ -48,6 +47,18 @@ MUTATIONS = [
      "int64_t ref = tb->ver[r];", 0),
     ("message-staleness-off-by-one", "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k;",
      "int64_t ref = (rule->row_staleness == 0) ? tb->ver[r] : k + 1;", 0),
+    # decay strategies and Hop-BW
+    ("geometric-exponent-off-by-one", "for (int64_t i = 0; i < s; ++i) p = p * (double)rule->lambda;",
+     "for (int64_t i = 0; i <= s; ++i) p = p * (double)rule->lambda;", 0),
+    ("geometric-ignored", "if (rule->decay == 0) return 1.0f;", "if (rule->decay >= 0) return 1.0f;", 0),
+    ("row-weight-not-applied", "S[r * d + j] += (double)fo * (double)gm[i * d + j];",
+     "S[r * d + j] += (double)gm[i * d + j];", 0),
+    ("dense-weight-not-applied", "if (f[m] > 0.0f) S += (double)f[m] * (double)dense_grads[m][e];",
+     "if (f[m] > 0.0f) S += (double)dense_grads[m][e];", 0),
+    ("hopbw-drops-earliest", "if (m >= M - rule->drop_latest) return 0.0f;",
+     "if (m < rule->drop_latest) return 0.0f;", 0),
+    ("hopbw-off-by-one", "if (m >= M - rule->drop_latest) return 0.0f;",
+     "if (m > M - rule->drop_latest) return 0.0f;", 0),
 ]
 
 
