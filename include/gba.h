@@ -78,11 +78,20 @@ typedef struct {
  *   sparse_denominator 0: divide a row's kept sum by the number of messages in
  *                 the global batch that contain the row (Alg. 2 "workers that
  *                 encountered the particular ID"), 1: by the kept ones, 2: by M.
+ *   decay 0: a kept gradient weighs 1 (Eq. (1) as printed);
+ *         1: a kept gradient of staleness s weighs lambda^s (Sec. 4.1 allows
+ *            other decay strategies; lambda^s is s products in double, rounded
+ *            to float once); needs 0 < lambda <= 1 and iota <= 1023.
+ *   drop_latest: Hop-BW's backup workers (Sec. 5.1): the last drop_latest
+ *            popped messages of every step weigh 0 (dense and rows); 0: none.
  * iota = INT32_MAX keeps every gradient (BSP). */
 typedef struct {
   int32_t iota;
   int32_t row_staleness;
   int32_t sparse_denominator;
+  int32_t decay;
+  float lambda;
+  int32_t drop_latest;
 } gba_staleness_desc;
 
 /* The sparse part of one message for one table: n ids and n x dim gradient rows
@@ -130,7 +139,8 @@ typedef struct {
  * global_batch       G: a step is applied once the buffered local batches sum to >= G
  *                    (Sec. 4.1: G_a = B_a * M equals the synchronous B_s * N_s).
  * max_buffered_msgs  capacity of the gradient buffer, in messages (>= 1).
- * st                 staleness rule (NULL: iota = INT32_MAX, tags, encountered).
+ * st                 staleness rule (NULL: iota = INT32_MAX, tags, encountered,
+ *                    weight 1, nothing ignored).
  * init_seed          weights are initialised from a counter-based hash of
  *                    (seed, table, element); optimizer state from the descriptors.
  * cuda_stream        cudaStream_t for all work of the handle; NULL makes a new one.
@@ -252,6 +262,26 @@ gba_status gba_token_list_create(int64_t repeats, int32_t workers, gba_token_lis
 gba_status gba_fetch_token(gba_token_list* tl, int64_t* token);
 gba_status gba_token_list_state(gba_token_list* tl, int64_t* queued, int64_t* fetched);
 void gba_token_list_destroy(gba_token_list* tl);
+
+/*
+ * gba_set_eager_dense - when on, a pushed message's dense gradient is added to
+ * the compensated sum of the global step it belongs to at push time, instead
+ * of being kept until that step (the memory saving of the paper's Alg. 2
+ * discussion: the weighted sum over some gradients can be executed in
+ * advance, based on the tokens).  The FIFO fixes each message's step (the
+ * shortest prefix of buffered local batches reaching G), so its weight
+ * (Eq. (1) or the decay strategy) is known when it arrives.  Sums are formed
+ * in arrival order, the order of the buffered mode, so results are identical.
+ * The dense part of the gradient buffer shrinks from one gradient per
+ * buffered message to one accumulator pair per pending global step (at most 8
+ * pending steps: a push that would need a ninth returns GBA_E_FULL).  Row
+ * gradients stay buffered (their decay needs the per-ID tags as of their
+ * step).  Only while no message is buffered (else GBA_E_STATE); GBA_E_ARG with
+ * drop_latest > 0, since the latest messages of a step are unknown at push.
+ * Pushes then launch a kernel on the handle's stream; push_ref's dense buffer
+ * may be reused once that kernel has run.
+ */
+gba_status gba_set_eager_dense(gba_handle* h, int32_t on);
 
 /*
  * gba_join - order the handle's stream after every step enqueued so far (their

@@ -53,7 +53,8 @@ class gba_table_desc(ctypes.Structure):
 
 class gba_staleness_desc(ctypes.Structure):
     _fields_ = [("iota", ctypes.c_int32), ("row_staleness", ctypes.c_int32),
-                ("sparse_denominator", ctypes.c_int32)]
+                ("sparse_denominator", ctypes.c_int32), ("decay", ctypes.c_int32),
+                ("lambda_", ctypes.c_float), ("drop_latest", ctypes.c_int32)]
 
 
 class gba_sparse_grad(ctypes.Structure):
@@ -100,6 +101,7 @@ _SIGNATURES = {
     "gba_set_debug": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_set_overlap": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_join": (ctypes.c_int, [_P]),
+    "gba_set_eager_dense": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_pull": (ctypes.c_int, [_P, ctypes.c_int32, _P, ctypes.c_int64, _P]),
     "gba_token_list_create": (ctypes.c_int, [ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(_P)]),
     "gba_fetch_token": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int64)]),
@@ -223,7 +225,8 @@ class GBA:
     """One parameter-server state on the current CUDA device."""
 
     def __init__(self, tables, dense_size, dense_opt, global_batch, max_buffered_msgs,
-                 iota=INT32_MAX, row_staleness=0, sparse_denominator=0, seed=0, stream=None):
+                 iota=INT32_MAX, row_staleness=0, sparse_denominator=0, seed=0, stream=None,
+                 decay=0, lam=1.0, drop_latest=0):
         """tables: list of (rows, dim, id_mode, max_ids_per_msg, gba_opt_desc)."""
         import torch
         self.torch = torch
@@ -234,7 +237,8 @@ class GBA:
         self.D = int(dense_size)
         self.dense_opt = dense_opt
         descs = [gba_table_desc(int(r), int(d), int(m), int(mx), o) for (r, d, m, mx, o) in tables]
-        st = gba_staleness_desc(int(iota), int(row_staleness), int(sparse_denominator))
+        st = gba_staleness_desc(int(iota), int(row_staleness), int(sparse_denominator),
+                                int(decay), float(lam), int(drop_latest))
         if stream is None:
             stream = torch.cuda.current_stream()
         self.stream = stream
@@ -343,6 +347,9 @@ class GBA:
                               ids.numel(), out.data_ptr() if ids.numel() else None),
               self.h, "gba_pull")
         return out
+
+    def set_eager_dense(self, on=True):
+        check(self.L.gba_set_eager_dense(self.h, int(on)), self.h, "gba_set_eager_dense")
 
     def join(self):
         """Order the handle's stream after every step enqueued so far."""

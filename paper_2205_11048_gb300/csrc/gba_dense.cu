@@ -128,15 +128,30 @@ __global__ void __launch_bounds__(DENSE_THREADS)
           aborted = true;
           break;
         }
+        if (a.decay == 0) {
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          if (mine[h]) {
-            const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT +
-                                                              h * HALF + 4 * c);
-            csum_add(acc[4 * h + 0], v.x);
-            csum_add(acc[4 * h + 1], v.y);
-            csum_add(acc[4 * h + 2], v.z);
-            csum_add(acc[4 * h + 3], v.w);
+          for (int h = 0; h < 2; ++h) {
+            if (mine[h]) {
+              const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT +
+                                                                h * HALF + 4 * c);
+              csum_add(acc[4 * h + 0], v.x);
+              csum_add(acc[4 * h + 1], v.y);
+              csum_add(acc[4 * h + 2], v.z);
+              csum_add(acc[4 * h + 3], v.w);
+            }
+          }
+        } else {  // weighted: f_m * g with the product's rounding error kept
+          const float f = sc.fw[j];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            if (mine[h]) {
+              const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT +
+                                                                h * HALF + 4 * c);
+              csum_add_prod(acc[4 * h + 0], f, v.x);
+              csum_add_prod(acc[4 * h + 1], f, v.y);
+              csum_add_prod(acc[4 * h + 2], f, v.z);
+              csum_add_prod(acc[4 * h + 3], f, v.w);
+            }
           }
         }
         __syncwarp();
@@ -162,7 +177,8 @@ __global__ void __launch_bounds__(DENSE_THREADS)
     if (blockIdx.x == 0 && c < (int)(da.D - D4)) {
       const int64_t e = D4 + c;
       CSum acc{0.f, 0.f};
-      for (int j = 0; j < n_kept; ++j) csum_add(acc, a.dense_ptr[sc.kept_list[j]][e]);
+      for (int j = 0; j < n_kept; ++j)
+        csum_add_prod(acc, a.decay == 0 ? 1.f : sc.fw[j], a.dense_ptr[sc.kept_list[j]][e]);
       float wv = da.w[e], a0 = da.s0[e], a1 = da.opt.kind == 1 ? da.s1[e] : 0.f;
       opt_update(da.opt, wv, a0, a1, __fdiv_rn(csum_value(acc), Mf));
       da.w[e] = wv;
@@ -171,6 +187,65 @@ __global__ void __launch_bounds__(DENSE_THREADS)
     }
   }
   __syncthreads();
+}
+
+// ---------------------------------------------------------------------------
+// Eager aggregation (Alg. 2 discussion: the weighted sum of the gradients can
+// be executed in advance, based on the tokens).  Under the FIFO every pushed
+// message belongs to a known future step, so its weight is known at push: its
+// dense gradient is added to that step's compensated accumulator (hi, lo)
+// right away, in push order -- the order the buffered K5 sums in -- and the
+// step then reads D accumulators instead of its kept messages.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256)
+    k_dense_accumulate(float* __restrict__ hi, float* __restrict__ lo,
+                       const float* __restrict__ g, int64_t D, float f, int first) {
+  const int64_t D4 = D & ~3ll;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < D4 / 4; q += stride) {
+    const float4 v = reinterpret_cast<const float4*>(g)[q];
+    const float x[4] = {v.x, v.y, v.z, v.w};
+    float4 h4 = make_float4(0.f, 0.f, 0.f, 0.f), l4 = h4;
+    if (!first) {
+      h4 = reinterpret_cast<const float4*>(hi)[q];
+      l4 = reinterpret_cast<const float4*>(lo)[q];
+    }
+    float hh[4] = {h4.x, h4.y, h4.z, h4.w}, ll[4] = {l4.x, l4.y, l4.z, l4.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      CSum c{hh[i], ll[i]};
+      csum_add_prod(c, f, x[i]);
+      hh[i] = c.hi;
+      ll[i] = c.lo;
+    }
+    reinterpret_cast<float4*>(hi)[q] = make_float4(hh[0], hh[1], hh[2], hh[3]);
+    reinterpret_cast<float4*>(lo)[q] = make_float4(ll[0], ll[1], ll[2], ll[3]);
+  }
+  if (blockIdx.x == 0 && threadIdx.x < (int)(D - D4)) {
+    const int64_t e = D4 + threadIdx.x;
+    CSum c{first ? 0.f : hi[e], first ? 0.f : lo[e]};
+    csum_add_prod(c, f, g[e]);
+    hi[e] = c.hi;
+    lo[e] = c.lo;
+  }
+}
+
+// The step's dense update from its accumulator (has_sum 0: no message was
+// kept, the gradient is 0).
+__global__ void __launch_bounds__(256)
+    k_dense_apply_eager(DenseArgs da, const float* __restrict__ hi, const float* __restrict__ lo,
+                        int has_sum, ErrSink err) {
+  if (__syncthreads_or((*(volatile uint32_t*)err.step & (ERR_ID_RANGE | ERR_TIMEOUT)) != 0u)) return;
+  const float Mf = (float)da.M;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < da.D; e += stride) {
+    const float v = has_sum ? __fadd_rn(hi[e], lo[e]) : 0.f;
+    float w = da.w[e], s0 = da.s0[e], s1 = da.opt.kind == 1 ? da.s1[e] : 0.f;
+    opt_update(da.opt, w, s0, s1, __fdiv_rn(v, Mf));
+    da.w[e] = w;
+    da.s0[e] = s0;
+    if (da.opt.kind == 1) da.s1[e] = s1;
+  }
 }
 
 }  // namespace
@@ -190,6 +265,22 @@ void launch_dense(const StepArgs& a, const DenseArgs& da, StepScratch sc, ErrSin
   if (grid > n_tiles) grid = n_tiles;
   if (grid < 1) grid = 1;
   k_dense_apply<<<(unsigned)grid, DENSE_THREADS, smem, s>>>(a, da, sc, err, wait_ns);
+}
+
+void launch_dense_accumulate(float* hi, float* lo, const float* g, int64_t D, float f, bool first,
+                             int num_sms, cudaStream_t s) {
+  int64_t grid = (D / 4 + 255) / 256;
+  if (grid > (int64_t)num_sms * 8) grid = (int64_t)num_sms * 8;
+  if (grid < 1) grid = 1;
+  k_dense_accumulate<<<(unsigned)grid, 256, 0, s>>>(hi, lo, g, D, f, first ? 1 : 0);
+}
+
+void launch_dense_eager(const DenseArgs& da, const float* hi, const float* lo, bool has_sum,
+                        ErrSink err, int num_sms, cudaStream_t s) {
+  int64_t grid = (da.D + 255) / 256;
+  if (grid > (int64_t)num_sms * 8) grid = (int64_t)num_sms * 8;
+  if (grid < 1) grid = 1;
+  k_dense_apply_eager<<<(unsigned)grid, 256, 0, s>>>(da, hi, lo, has_sum ? 1 : 0, err);
 }
 
 }  // namespace gba

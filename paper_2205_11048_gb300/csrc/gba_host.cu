@@ -23,6 +23,8 @@ constexpr int MAX_DIM = 256;
 constexpr int META_SLOTS = 4;
 constexpr int MAX_PASSES = 4;
 constexpr int64_t MAX_STEP_OCC = (1ll << 30) - 1;
+constexpr int MAX_WTAB = 1024;  // decay weights lambda^s for s < MAX_WTAB
+constexpr int EAGER_SLOTS = 8;  // pending global steps with eager dense accumulators
 // Per-step buffers exist twice, so that step k + 1's message weights and sort
 // run (on the sort stream) while step k's segment-sum and dense update run.
 constexpr int SLOTS = 2;
@@ -142,6 +144,24 @@ struct gba_handle {
   uint32_t* d_seg_total = nullptr;         // [T] rows of each table in the last step
   int d_max = 1;
 
+  float* d_wtab = nullptr;    // decay weights lambda^s (decay 1)
+  int32_t n_wtab = 0;
+  std::vector<float> h_wtab;
+
+  // eager dense aggregation: one compensated accumulator (hi, lo) per pending
+  // global step, filled at push time
+  bool eager = false;
+  struct EagerGroup {
+    int64_t accB;  // local batches of the step's messages so far
+    int slot;      // its accumulator
+    bool has_sum;  // some message of the step was kept
+  };
+  std::deque<EagerGroup> egroups;
+  int n_acc = 0;
+  float* d_acc = nullptr;          // [n_acc][2][D_pad]
+  cudaEvent_t acc_ev[EAGER_SLOTS] = {};
+  bool acc_ev_set[EAGER_SLOTS] = {};
+  float* d_stage_dense = nullptr;  // copying pushes stage the dense gradient here
   uint32_t* d_err = nullptr;
   uint32_t* h_err = nullptr;  // mapped pinned
   ErrSink sink{};
@@ -294,6 +314,11 @@ void free_all(gba_handle* h) {
                   (void*)h->d_part_hi, (void*)h->d_part_lo, (void*)h->d_seg_total})
     cudaFree(p);
   cudaFree(h->d_err);
+  cudaFree(h->d_wtab);
+  cudaFree(h->d_acc);
+  cudaFree(h->d_stage_dense);
+  for (cudaEvent_t e : h->acc_ev)
+    if (e) cudaEventDestroy(e);
   if (h->h_err) cudaFreeHost(h->h_err);
   cudaFree(h->d_stats);
   for (auto& p : h->pending) {
@@ -424,6 +449,16 @@ gba_status ensure_arenas(gba_handle* h) {
   return GBA_OK;
 }
 
+// The dense weight of a message with this token applied at step k_apply
+// (Eq. (1), or the decay strategy; the same numbers the kernels use).
+float message_weight(const gba_handle* h, int64_t k_apply, int64_t token) {
+  const int64_t diff = k_apply - token;
+  const int64_t s = diff > 0 ? diff : 0;
+  if (s > (int64_t)h->st.iota) return 0.f;
+  if (h->st.decay == 0) return 1.f;
+  return s < (int64_t)h->h_wtab.size() ? h->h_wtab[s] : 0.f;
+}
+
 gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_table,
                        const float* dense_grad, int32_t local_batch, bool copy) {
   if (!h) return GBA_E_ARG;
@@ -448,6 +483,18 @@ gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_
   if (!copy && h->D > 0 && ((uintptr_t)dense_grad & 15u) != 0)
     return set_err(h, GBA_E_ARG, "dense_grad not 16-byte aligned");
   if ((int64_t)h->fifo.size() >= h->max_buf) return set_err(h, GBA_E_FULL, "gradient buffer full");
+  const bool eager = h->eager && h->D > 0;
+  // eager: the step this message belongs to, and its accumulator
+  const bool new_group = eager && (h->egroups.empty() || h->egroups.back().accB >= h->G);
+  int new_slot = -1;
+  if (new_group) {
+    bool held[EAGER_SLOTS] = {};
+    for (const auto& gr : h->egroups) held[gr.slot] = true;
+    for (int i = 0; i < h->n_acc && new_slot < 0; ++i)
+      if (!held[i]) new_slot = i;
+    if (new_slot < 0)
+      return set_err(h, GBA_E_FULL, "every eager accumulator holds a pending global step");
+  }
 
   Msg m;
   m.token = token;
@@ -462,7 +509,7 @@ gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_
     if (s != GBA_OK) return s;
     // The copy may overwrite buffer space of messages that earlier steps read.
     if (h->overlap) join_steps(h);
-    if (h->D > 0 && h->slot_count >= h->max_buf)
+    if (h->D > 0 && !eager && h->slot_count >= h->max_buf)
       return set_err(h, GBA_E_FULL, "gradient buffer full");
     std::vector<int64_t> saved_tail(h->T);
     for (int t = 0; t < h->T; ++t) saved_tail[t] = h->tables[t].arena.vtail;
@@ -490,7 +537,7 @@ gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_
                                     n * dim * sizeof(float), cudaMemcpyDefault, h->stream));
       }
     }
-    if (h->D > 0) {
+    if (h->D > 0 && !eager) {
       const int32_t slot = (h->slot_head + h->slot_count) % h->max_buf;
       float* dst = h->dense_ring + (size_t)slot * h->D_pad;
       GBA_CUDA(h, cudaMemcpyAsync(dst, dense_grad, h->D * sizeof(float), cudaMemcpyDefault,
@@ -507,6 +554,29 @@ gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_
       m.n[t] = per_table[t].n;
     }
     m.dense = dense_grad;
+  }
+  if (eager) {  // the dense gradient joins its step's accumulator now
+    if (new_group) {
+      if (h->acc_ev_set[new_slot]) cudaStreamWaitEvent(h->stream, h->acc_ev[new_slot], 0);
+      h->egroups.push_back(gba_handle::EagerGroup{0, new_slot, false});
+    }
+    gba_handle::EagerGroup& gr = h->egroups.back();
+    const int64_t k_apply = h->k + (int64_t)h->egroups.size() - 1;
+    const float f = message_weight(h, k_apply, token);
+    if (f > 0.f) {
+      const float* src = dense_grad;
+      if (copy) {
+        GBA_CUDA(h, cudaMemcpyAsync(h->d_stage_dense, dense_grad, h->D * sizeof(float),
+                                    cudaMemcpyDefault, h->stream));
+        src = h->d_stage_dense;
+      }
+      float* hi = h->d_acc + (size_t)gr.slot * 2 * h->D_pad;
+      launch_dense_accumulate(hi, hi + h->D_pad, src, h->D, f, !gr.has_sum, h->num_sms, h->stream);
+      GBA_CUDA(h, cudaGetLastError());
+      gr.has_sum = true;
+    }
+    gr.accB += local_batch;
+    m.dense = nullptr;
   }
   h->fifo.push_back(std::move(m));
   return GBA_OK;
@@ -536,10 +606,14 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   }
   if (total_rows >= 0xFFFFFFFFull) return GBA_E_ARG;  // keys are 32-bit, one value reserved
   if (dense_size > 0 && validate_opt(*dense_opt) != GBA_OK) return GBA_E_ARG;
-  gba_staleness_desc rule{0x7FFFFFFF, 0, 0};
+  gba_staleness_desc rule{0x7FFFFFFF, 0, 0, 0, 1.0f, 0};
   if (st) rule = *st;
   if (rule.iota < 0 || (rule.row_staleness != 0 && rule.row_staleness != 1) ||
-      rule.sparse_denominator < 0 || rule.sparse_denominator > 2)
+      rule.sparse_denominator < 0 || rule.sparse_denominator > 2 ||
+      (rule.decay != 0 && rule.decay != 1) || rule.drop_latest < 0)
+    return GBA_E_ARG;
+  if (rule.decay == 1 &&
+      (!(rule.lambda > 0.f && rule.lambda <= 1.f) || rule.iota >= MAX_WTAB))
     return GBA_E_ARG;
 
   gba_handle* h = new (std::nothrow) gba_handle();
@@ -593,7 +667,8 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
     TableState& ts = h->tables[t];
     ts.desc = tables[t];
     ts.key_base = base;
-    h->h_tinfo[t] = TableInfo{tables[t].rows, base, tables[t].id_mode};
+    h->h_tinfo[t] = TableInfo{tables[t].rows, base, tables[t].id_mode,
+                              ~0ull / (uint64_t)tables[t].rows};
     base += (uint32_t)tables[t].rows;
     h->d_max = std::max(h->d_max, (int)tables[t].dim);
   }
@@ -670,6 +745,20 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
     }
   }
   if (!dev_alloc((void**)&h->d_seg_total, (size_t)std::max(h->T, 1) * 4)) return fail(GBA_E_OOM);
+  if (rule.decay == 1) {  // lambda^s as s products in double, rounded once, s = 0 .. iota
+    h->n_wtab = rule.iota + 1;
+    std::vector<float>& wt = h->h_wtab;
+    wt.resize(h->n_wtab);
+    double pw = 1.0;
+    for (int32_t s2 = 0; s2 < h->n_wtab; ++s2) {
+      wt[s2] = (float)pw;
+      pw = pw * (double)rule.lambda;
+    }
+    if (!dev_alloc((void**)&h->d_wtab, wt.size() * sizeof(float))) return fail(GBA_E_OOM);
+    if (cudaMemcpy(h->d_wtab, wt.data(), wt.size() * sizeof(float), cudaMemcpyHostToDevice) !=
+        cudaSuccess)
+      return fail(GBA_E_CUDA);
+  }
   if (!dev_alloc((void**)&h->d_err, 4) || !dev_alloc((void**)&h->d_stats, sizeof(DevStats)))
     return fail(GBA_E_OOM);
   if (cudaHostAlloc((void**)&h->h_err, 4, cudaHostAllocMapped) != cudaSuccess)
@@ -811,6 +900,10 @@ int32_t gba_try_apply(gba_handle* h) {
   a.iota = h->st.iota;
   a.row_staleness = h->st.row_staleness;
   a.sparse_den = h->st.sparse_denominator;
+  a.decay = h->st.decay;
+  a.drop_latest = h->st.drop_latest;
+  a.n_wtab = h->n_wtab;
+  a.wtab = h->d_wtab;
   a.tokens = (const int64_t*)(dmeta + o_tok);
   a.dense_ptr = (const float* const*)(dmeta + o_dense);
   a.msg_off = (const uint32_t*)(dmeta + o_off);
@@ -834,7 +927,17 @@ int32_t gba_try_apply(gba_handle* h) {
     DenseArgs da{h->dw, h->ds0, h->ds1, h->D, M, make_opt_step(h->dense_opt, p1, p2)};
     cudaEventRecord(h->ev_hist[b], h->sorts);
     cudaStreamWaitEvent(h->side, h->ev_hist[b], 0);
-    {
+    if (h->eager) {  // the step's sum was accumulated at push time
+      const gba_handle::EagerGroup gr = h->egroups.front();
+      h->egroups.pop_front();
+      const float* hi = h->d_acc + (size_t)gr.slot * 2 * h->D_pad;
+      {
+        Timed tm(h, GBA_K_DENSE, h->side);
+        launch_dense_eager(da, hi, hi + h->D_pad, gr.has_sum, sink, h->num_sms, h->side);
+      }
+      cudaEventRecord(h->acc_ev[gr.slot], h->side);
+      h->acc_ev_set[gr.slot] = true;
+    } else {
       Timed tm(h, GBA_K_DENSE, h->side);
       launch_dense(a, da, sc, sink, h->wait_ns, h->num_sms, h->side);
     }
@@ -946,7 +1049,7 @@ int32_t gba_try_apply(gba_handle* h) {
     if (m.copied) {
       for (int t = 0; t < T; ++t)
         if (m.n[t] > 0) h->tables[t].arena.release_through(m.arena_v[t] + m.n[t]);
-      if (h->D > 0) {
+      if (h->D > 0 && m.dense != nullptr) {  // a dense ring slot (not eager)
         h->slot_head = (h->slot_head + 1) % h->max_buf;
         h->slot_count--;
       }
@@ -1051,9 +1154,27 @@ gba_status gba_pull(gba_handle* h, int32_t t, const int64_t* ids, int64_t n, flo
   const TableState& ts = h->tables[t];
   ErrSink sink = h->sink;
   sink.step = h->d_err;  // no step of its own: the handle's word takes both roles
-  launch_pull_rows(ts.w, ts.desc.rows, ts.desc.dim, ts.desc.id_mode, ids, n, out, sink,
-                   h->num_sms, h->stream);
+  launch_pull_rows(ts.w, ts.desc.rows, ts.desc.dim, ts.desc.id_mode, h->h_tinfo[t].mod_magic, ids,
+                   n, out, sink, h->num_sms, h->stream);
   GBA_CUDA(h, cudaGetLastError());
+  return GBA_OK;
+}
+
+gba_status gba_set_eager_dense(gba_handle* h, int32_t on) {
+  if (!h) return GBA_E_ARG;
+  if (h->failed) return set_err(h, GBA_E_STATE, "handle failed earlier");
+  if (!h->fifo.empty()) return set_err(h, GBA_E_STATE, "messages are buffered");
+  if (on && h->st.drop_latest > 0)
+    return set_err(h, GBA_E_ARG, "eager aggregation cannot know the latest messages of a step");
+  cudaSetDevice(h->device);
+  if (on && h->D > 0 && !h->d_acc) {
+    h->n_acc = std::min(EAGER_SLOTS, std::max(1, (int)h->max_buf));
+    GBA_CUDA(h, cudaMalloc(&h->d_acc, (size_t)h->n_acc * 2 * h->D_pad * sizeof(float)));
+    GBA_CUDA(h, cudaMalloc(&h->d_stage_dense, (size_t)h->D_pad * sizeof(float)));
+    for (int i = 0; i < h->n_acc; ++i)
+      GBA_CUDA(h, cudaEventCreateWithFlags(&h->acc_ev[i], cudaEventDisableTiming));
+  }
+  h->eager = on != 0;
   return GBA_OK;
 }
 

@@ -91,7 +91,20 @@ struct TableInfo {
   int64_t V;
   uint32_t key_base;  // first global key of the table
   int32_t id_mode;    // 0 DIRECT, 1 MODULO
+  uint64_t mod_magic; // floor((2^64 - 1) / V), for mod_u64
 };
+
+// x mod V for a 64-bit x and V < 2^32, without a 64-bit division: the
+// quotient estimate floor(x * m / 2^64) with m = floor((2^64 - 1) / V) is at
+// most 2 below floor(x / V) (division by an invariant integer through a
+// precomputed reciprocal, after Granlund and Montgomery 1994), so at most two
+// corrections give the exact remainder.
+__device__ __forceinline__ uint64_t mod_u64(uint64_t x, uint64_t V, uint64_t m) {
+  uint64_t r = x - __umul64hi(x, m) * V;
+  if (r >= V) r -= V;
+  if (r >= V) r -= V;
+  return r;
+}
 
 // ---- optimizer parameters of one parameter group for one step ---------------
 struct OptStep {
@@ -327,6 +340,13 @@ cudaError_t configure_dense();
 void launch_dense(const StepArgs& a, const DenseArgs& da, StepScratch sc, ErrSink err,
                   int64_t wait_ns, int num_sms, cudaStream_t s);
 
+// Eager dense aggregation: add f * g to a step's accumulator (first: start it),
+// and the step's update from the accumulator.
+void launch_dense_accumulate(float* hi, float* lo, const float* g, int64_t D, float f, bool first,
+                             int num_sms, cudaStream_t s);
+void launch_dense_eager(const DenseArgs& da, const float* hi, const float* lo, bool has_sum,
+                        ErrSink err, int num_sms, cudaStream_t s);
+
 void launch_init_table(float* w, float* s0, float* s1, int32_t* ver, int64_t rows, int32_t d,
                        int32_t kind, float init_acc, uint64_t seed, uint64_t tag,
                        cudaStream_t s);
@@ -337,8 +357,9 @@ void launch_init_dense(float* w, float* s0, float* s1, int64_t D, int32_t kind, 
 int launch_wait_selftest(int64_t limit_ns, cudaStream_t s, uint32_t* d_word, uint32_t* result);
 
 // Rows of one table for n ids (pull responding), into out[n][d].
-void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, const int64_t* ids, int64_t n,
-                      float* out, ErrSink err, int num_sms, cudaStream_t s);
+void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, uint64_t mod_magic,
+                      const int64_t* ids, int64_t n, float* out, ErrSink err, int num_sms,
+                      cudaStream_t s);
 
 // Compute capability (major * 10 + minor) of the device code the library's
 // kernels were loaded from on the current device, or -1.

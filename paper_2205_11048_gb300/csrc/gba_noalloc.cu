@@ -45,7 +45,8 @@ constexpr size_t kOffMsgOff = kOffTiles + 16;
 constexpr size_t kOffIdsPtr = kOffMsgOff + 16;
 constexpr size_t kOffNbase = kOffIdsPtr + 16;
 constexpr size_t kOffTinfo = kOffNbase + 16;
-constexpr size_t kOffErr = kOffTinfo + 32;
+constexpr size_t kOffErr = kOffTinfo + 32;  // TableInfo is 24 bytes
+static_assert(sizeof(gba::TableInfo) <= 32, "TableInfo outgrew its scratch slot");
 constexpr size_t kBytes = kOffErr + 16;
 static_assert(kBytes == GBA_STATIC_SORT_BYTES, "scratch size differs from the header");
 
@@ -76,6 +77,7 @@ __global__ void k_static_setup(unsigned char* base, const int64_t* ids, int64_t 
     ti->V = rows;
     ti->key_base = 0u;
     ti->id_mode = id_mode;
+    ti->mod_magic = ~0ull / (uint64_t)rows;
     uint32_t* err = reinterpret_cast<uint32_t*>(base + kOffErr);
     err[0] = 0u;
     err[1] = 0u;

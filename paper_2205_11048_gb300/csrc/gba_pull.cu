@@ -17,7 +17,7 @@ constexpr int PULL_THREADS = 256;
 
 template <bool VEC>
 __global__ void __launch_bounds__(PULL_THREADS)
-    k_pull_rows(const float* __restrict__ w, int64_t V, int d, int id_mode,
+    k_pull_rows(const float* __restrict__ w, int64_t V, int d, int id_mode, uint64_t mod_magic,
                 const int64_t* __restrict__ ids, int64_t n, float* __restrict__ out, int lg,
                 ErrSink err) {
   const int L = 1 << lg;
@@ -33,7 +33,7 @@ __global__ void __launch_bounds__(PULL_THREADS)
       ok = id >= 0 && id < V;
       row = ok ? (uint64_t)id : 0ull;
     } else {
-      row = (uint64_t)id % (uint64_t)V;
+      row = mod_u64((uint64_t)id, (uint64_t)V, mod_magic);
     }
     if (!ok && l == 0) raise_error(err, ERR_ID_RANGE);
     const float* src = w + row * (uint64_t)d;
@@ -53,8 +53,9 @@ __global__ void __launch_bounds__(PULL_THREADS)
 
 }  // namespace
 
-void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, const int64_t* ids, int64_t n,
-                      float* out, ErrSink err, int num_sms, cudaStream_t s) {
+void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, uint64_t mod_magic,
+                      const int64_t* ids, int64_t n, float* out, ErrSink err, int num_sms,
+                      cudaStream_t s) {
   if (n <= 0) return;
   const bool vec = (d & 3) == 0 && ((uintptr_t)out & 15u) == 0;
   const int pieces = vec ? d / 4 : d;
@@ -65,10 +66,10 @@ void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, const int64
   const int64_t cap = (int64_t)num_sms * 8;
   if (grid > cap) grid = cap;
   if (vec)
-    k_pull_rows<true><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, ids, n, out, lg, err);
+    k_pull_rows<true><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, mod_magic, ids, n, out, lg, err);
   else
-    k_pull_rows<false><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, ids, n, out, lg,
-                                                               err);
+    k_pull_rows<false><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, mod_magic, ids, n,
+                                                               out, lg, err);
 }
 
 }  // namespace gba

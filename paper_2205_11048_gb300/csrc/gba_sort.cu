@@ -92,7 +92,7 @@ __device__ __forceinline__ uint32_t occurrence_key(const StepArgs& a, const uint
       row = (uint64_t)id;
     }
   } else {
-    row = (uint64_t)id % (uint64_t)ti.V;
+    row = mod_u64((uint64_t)id, (uint64_t)ti.V, ti.mod_magic);
   }
   return ti.key_base + (uint32_t)row;
 }
@@ -136,14 +136,21 @@ __global__ void __launch_bounds__(256) k_message_weights(StepArgs a, StepScratch
     const int m = base + lane;
     int keep = 0;
     unsigned long long s = 0;
+    float f = 0.f;
     if (m < a.M) {
       const int64_t diff = a.k - a.tokens[m];
       s = diff > 0 ? (unsigned long long)diff : 0ull;
-      keep = (s <= (unsigned long long)(int64_t)a.iota) ? 1 : 0;
+      // Eq. (1) (or the decay strategy), and Hop-BW's ignored latest messages
+      f = m < a.M - a.drop_latest ? decay_weight(a, s) : 0.f;
+      keep = f > 0.f ? 1 : 0;
       sc.keep[m] = keep;
     }
     const uint32_t b = __ballot_sync(0xffffffffu, keep != 0);
-    if (keep) sc.kept_list[kept + __popc(b & lanemask_lt())] = m;
+    if (keep) {
+      const int j = kept + __popc(b & lanemask_lt());
+      sc.kept_list[j] = m;
+      if (sc.fw) sc.fw[j] = f;
+    }
     kept += __popc(b);
     s_sum += s;
     s_max = s > s_max ? s : s_max;

@@ -64,6 +64,11 @@ def _create(L, tables, D=8, G=4, max_buf=4, st=None, dense_opt=None):
     dict(tables=[_table()], st=B.gba_staleness_desc(-1, 0, 0)),
     dict(tables=[_table()], st=B.gba_staleness_desc(1, 2, 0)),
     dict(tables=[_table()], st=B.gba_staleness_desc(1, 0, 3)),
+    dict(tables=[_table()], st=B.gba_staleness_desc(1, 0, 0, 2, 1.0, 0)),
+    dict(tables=[_table()], st=B.gba_staleness_desc(1, 0, 0, 1, 0.0, 0)),
+    dict(tables=[_table()], st=B.gba_staleness_desc(1, 0, 0, 1, 1.5, 0)),
+    dict(tables=[_table()], st=B.gba_staleness_desc(1024, 0, 0, 1, 0.5, 0)),
+    dict(tables=[_table()], st=B.gba_staleness_desc(1, 0, 0, 0, 1.0, -1)),
     dict(tables=[_table()], dense_opt=B.opt_desc(1, 0.01, 0.1, 1.0, 0.999, 1e-8)),
 ])
 def test_create_rejects_bad_arguments(L, bad):

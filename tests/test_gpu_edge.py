@@ -134,6 +134,67 @@ def test_rule_option_goldens_exactly(variant):
     g.close()
 
 
+@pytest.mark.parametrize("name", ["geometric", "hop_bw"])
+def test_decay_variant_goldens_exactly(name):
+    """The hand-worked steps of geometric decay (lambda^s) and Hop-BW's ignored
+    latest gradients, through the CUDA path: exact values."""
+    from tests import _pins
+    gj = _pins.load_golden()["decay_variants"]
+    var = gj[name]
+    F = _pins.F
+    lr, acc0 = F(gj["table"]["lr"]), F(gj["table"]["init_acc"])
+    tables = [(4, 2, 0, 8, B.opt_desc(0, lr, acc0))]
+    g = B.GBA(tables, 2, B.opt_desc(0, lr, acc0), var["global_batch"], 8, seed=4321,
+              **var["rule"])
+    w0 = g.table(0)[0].cpu().numpy().astype(np.float64)
+    dw0 = g.dense()[0].cpu().numpy().astype(np.float64)
+    for step in var["steps"]:
+        for m in step["messages"]:
+            ids = torch.tensor(m["ids"], dtype=torch.int64, device="cuda")
+            rows = torch.tensor(m["rows"], dtype=torch.float32, device="cuda")
+            g.push(m["token"], [ids], [rows], torch.tensor(m["dense"], dtype=torch.float32,
+                                                           device="cuda"), m["B"])
+        assert g.try_apply() == 1
+        e = step["expect"]
+        assert g.keep().tolist() == e["keep"]
+        w, s0, _, ver = g.table(0)
+        for r in range(4):
+            assert (w[r].cpu().numpy().astype(np.float64) - w0[r]).tolist() == \
+                [F(v) for v in e["dw"][str(r)]]
+            assert s0[r].cpu().numpy().astype(np.float64).tolist() == \
+                [F(v) for v in e["acc"][str(r)]]
+        assert ver.cpu().tolist() == e["ver"]
+        dw, ds0, _ = g.dense()
+        assert (dw.cpu().numpy().astype(np.float64) - dw0).tolist() == \
+            [F(v) for v in e["dense_dw"]]
+        assert ds0.cpu().numpy().astype(np.float64).tolist() == [F(v) for v in e["dense_acc"]]
+    g.close()
+
+
+@pytest.mark.parametrize("rule", [dict(iota=6, decay=1, lam=0.7),
+                                  dict(iota=3, decay=1, lam=0.5, row_staleness=1),
+                                  dict(iota=O.INT32_MAX, drop_latest=1),
+                                  dict(iota=2, decay=1, lam=0.9, drop_latest=2,
+                                       sparse_denominator=1)])
+@pytest.mark.parametrize("kind", [0, 1])
+def test_decay_variants_against_the_oracle(rule, kind):
+    """Geometric decay and Hop-BW on a random stream with stale tokens, hot
+    rows (long rows) and two row widths, Adagrad and Adam."""
+    rng = np.random.default_rng(17 + kind)
+    cfg = cfg_of([(500, 16, 0, kind), (300, 6, 0, kind)], D=1031, G=6, dense_kind=kind)
+    steps = []
+    for k in range(5):
+        batch = []
+        for m in range(6):
+            n0 = int(rng.integers(0, 400))
+            ids0 = np.concatenate([rng.zipf(1.4, n0) % 500, np.full(int(rng.integers(0, 90)), 7)])
+            ids1 = rng.integers(0, 300, int(rng.integers(0, 50)))
+            tok = max(0, k - int(rng.integers(0, 5)))
+            batch.append(msg(tok, [ids0, ids1], [16, 6], 1031))
+        steps.append(batch)
+    run_custom(cfg, steps, rule=rule)
+
+
 @pytest.mark.parametrize("dim", [1, 3, 4, 8, 19, 24, 64, 128, 200, 256])
 @pytest.mark.parametrize("kind", [0, 1])
 def test_row_widths_and_optimizers(dim, kind):
@@ -444,4 +505,74 @@ def test_pull_of_an_out_of_range_id_is_latched():
     assert np.all(o[1] == 0)
     w = _raw_table_w(g, 0).view(100, 8).cpu().numpy()
     assert np.array_equal(o[[0, 2]], w[[3, 5]])
+    g.close()
+
+
+@pytest.mark.parametrize("by_ref", [False, True])
+@pytest.mark.parametrize("rule", [dict(iota=2), dict(iota=5, decay=1, lam=0.8)])
+def test_eager_dense_equals_buffered(by_ref, rule):
+    """Eager push-time aggregation of the dense gradients gives the buffered
+    mode's state bit for bit, and matches the oracle, with varying local
+    batches (steps of different sizes, overshoot) and stale tokens."""
+    rng = np.random.default_rng(5 + by_ref)
+    cfg = cfg_of([(400, 8, 0, 0)], D=20_011, G=6, dense_kind=1)
+    stream = []
+    k_expected = 0
+    for k in range(6):
+        acc = 0
+        while acc < cfg.G:  # one step's messages: local batches summing to >= G
+            b = int(rng.integers(1, 4))
+            m = msg(max(0, k - int(rng.integers(0, 4))), [rng.integers(0, 400, 40)], [8], 20_011,
+                    B_=b)
+            stream.append(m)
+            acc += b
+    outs = []
+    for eager in (False, True):
+        tables = [(400, 8, 0, 4096, H.opt_desc(cfg.tables[0].opt))]
+        g = B.GBA(tables, cfg.D, H.opt_desc(cfg.dense_opt), cfg.G, 64, seed=cfg.seed, **rule)
+        if eager:
+            g.set_eager_dense(True)
+        orc = H.make_oracle(cfg, rule=rule)
+        n_steps = 0
+        for m in stream:
+            (g.push_ref if by_ref else g.push)(m["token"], m["ids"], m["rows"], m["dense"],
+                                               m["local_batch"])
+            orc.push(H.to_oracle(m))
+            a, c = g.try_apply(), orc.try_apply()
+            assert a == c
+            n_steps += a
+        g.sync()
+        H.compare_state(g, orc, H.TOL_ONE_STEP)
+        outs.append([t.cpu() for t in g.dense()[:3] if t is not None] + [g.table(0)[0].cpu()])
+        assert n_steps >= 6
+        g.close()
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+def test_eager_dense_refusals_and_capacity():
+    tables = [(100, 4, 0, 16, B.opt_desc())]
+    g = B.GBA(tables, 1000, B.opt_desc(1, 0.001), 4, 64, seed=1, iota=3, drop_latest=1)
+    with pytest.raises(B.GBAError) as e:
+        g.set_eager_dense(True)
+    assert e.value.status == B.GBA_E_ARG
+    g.close()
+    g = B.GBA(tables, 1000, B.opt_desc(1, 0.001), 4, 64, seed=1, iota=3)
+    m = msg(0, [[1, 2]], [4], 1000, B_=4)
+    g.push(m["token"], m["ids"], m["rows"], m["dense"], 4)
+    with pytest.raises(B.GBAError) as e:  # messages are buffered
+        g.set_eager_dense(True)
+    assert e.value.status == B.GBA_E_STATE
+    assert g.try_apply() == 1
+    g.set_eager_dense(True)
+    # each message fills a whole step: eight pending steps fit, a ninth does not
+    for i in range(8):
+        g.push(m["token"], m["ids"], m["rows"], m["dense"], 4)
+    rc = g.L.gba_push(g.h, 0, (B.gba_sparse_grad * 1)(*g._grads(m["ids"], m["rows"])),
+                      m["dense"].data_ptr(), 4)
+    assert rc == B.GBA_E_FULL
+    for i in range(8):
+        assert g.try_apply() == 1
+    assert g.try_apply() == 0
+    g.sync()
     g.close()
