@@ -43,10 +43,22 @@ typedef enum {
 
 typedef enum { GBA_ADAGRAD = 0, GBA_ADAM = 1 } gba_optimizer;
 
-/* id -> row mapping of a table (no hash table on this path):
+/* id -> row mapping of a table:
  * DIRECT: the id is the row and must satisfy 0 <= id < rows;
- * MODULO: row = (uint64_t)id % rows (hashing trick; colliding ids share a row). */
-typedef enum { GBA_ID_DIRECT = 0, GBA_ID_MODULO = 1 } gba_id_mode;
+ * MODULO: row = (uint64_t)id % rows (hashing trick; colliding ids share a row);
+ * HASH:   an expandable hash table of 64-bit ids (the paper's models run on
+ *         DeepRec's expandable hash tables, Sec. 5.1): every distinct id gets a
+ *         row of its own, created when the id is first pushed and initialised
+ *         from the id (element id * dim + j of the table's counter-based
+ *         stream), so an id's values do not depend on where it is stored.
+ *         `rows` is the initial capacity (rounded up to a power of two, at
+ *         least 1024, at most 2^30); the table doubles before a step that
+ *         could fill more than half of it.  The id INT64_MIN is reserved
+ *         (a step containing it fails with GBA_E_ID_RANGE).  The arrays of
+ *         gba_get_table are indexed by slot: use gba_table_capacity for their
+ *         size and gba_lookup_rows for the slot of an id; growth moves rows
+ *         and replaces the arrays, so take the pointers again after a step. */
+typedef enum { GBA_ID_DIRECT = 0, GBA_ID_MODULO = 1, GBA_ID_HASH = 2 } gba_id_mode;
 
 /* Optimizer of a table or of the dense parameters.  Table 1 of the paper names
  * Adagrad and Adam; the update rules are the textbook ones, one IEEE float
@@ -262,6 +274,17 @@ gba_status gba_token_list_create(int64_t repeats, int32_t workers, gba_token_lis
 gba_status gba_fetch_token(gba_token_list* tl, int64_t* token);
 gba_status gba_token_list_state(gba_token_list* tl, int64_t* queued, int64_t* fetched);
 void gba_token_list_destroy(gba_token_list* tl);
+
+/* gba_table_capacity - the rows the arrays of table t hold now (for a HASH
+ * table, its current number of slots). */
+gba_status gba_table_capacity(gba_handle* h, int32_t t, int64_t* rows);
+
+/* gba_lookup_rows - for a HASH table, the row (slot) of each of n device
+ * int64 ids into n device int64 (-1 for an id not in the table), on the
+ * handle's stream after every step enqueued so far.  GBA_E_ARG for other
+ * tables. */
+gba_status gba_lookup_rows(gba_handle* h, int32_t t, const int64_t* ids, int64_t n,
+                           int64_t* rows_out);
 
 /*
  * gba_set_eager_dense - when on, a pushed message's dense gradient is added to

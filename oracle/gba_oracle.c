@@ -50,7 +50,9 @@ typedef struct {
 typedef struct {
   int64_t V;              /* rows in the table */
   int32_t d;              /* row width */
-  int32_t id_mode;        /* 0: row = id (0 <= id < V), 1: row = (uint64)id mod V */
+  int32_t id_mode;        /* 0: row = id (0 <= id < V), 1: row = (uint64)id mod V,
+                             2: every distinct id is its own row (a hash table of
+                                ids); the tracked "rows" are then ids */
   gbao_opt opt;
   int64_t n_track;        /* number of tracked rows */
   const int64_t* track;   /* tracked rows, strictly increasing, in [0, V) */
@@ -311,8 +313,11 @@ int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens
         if (tb->id_mode == 0) {
           if (id < 0 || id >= tb->V) { err = 1; continue; }
           x = id;
-        } else {
+        } else if (tb->id_mode == 1) {
           x = (int64_t)((uint64_t)id % (uint64_t)tb->V);
+        } else {
+          if (id == INT64_MIN) { err = 1; continue; }  /* the reserved id */
+          x = id;
         }
         int64_t r = find_tracked(tb->track, nt, x);
         if (r < 0) continue;

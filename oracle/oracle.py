@@ -166,7 +166,7 @@ class TableSpec:
     rows: int
     dim: int
     opt: OptSpec = field(default_factory=OptSpec)
-    id_mode: int = 0   # 0: row = id, 1: row = uint64(id) mod rows
+    id_mode: int = 0   # 0: row = id, 1: row = uint64(id) mod rows, 2: each id its own row
 
 
 @dataclass

@@ -28,7 +28,7 @@ STATUS_NAMES = {0: "GBA_OK", -1: "GBA_E_ARG", -2: "GBA_E_ID_RANGE", -3: "GBA_E_O
                 -4: "GBA_E_CUDA", -5: "GBA_E_DEVICE_TIMEOUT", -6: "GBA_E_STATE",
                 -7: "GBA_E_FULL"}
 ADAGRAD, ADAM = 0, 1
-DIRECT, MODULO = 0, 1
+DIRECT, MODULO, HASH = 0, 1, 2
 INT32_MAX = 2**31 - 1
 KERNEL_NAMES = ["weights", "sort_hist", "sort_pass", "seg_scan", "row_long", "row_apply",
                 "dense", "init", "other"]
@@ -102,6 +102,8 @@ _SIGNATURES = {
     "gba_set_overlap": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_join": (ctypes.c_int, [_P]),
     "gba_set_eager_dense": (ctypes.c_int, [_P, ctypes.c_int32]),
+    "gba_table_capacity": (ctypes.c_int, [_P, ctypes.c_int32, ctypes.POINTER(ctypes.c_int64)]),
+    "gba_lookup_rows": (ctypes.c_int, [_P, ctypes.c_int32, _P, ctypes.c_int64, _P]),
     "gba_pull": (ctypes.c_int, [_P, ctypes.c_int32, _P, ctypes.c_int64, _P]),
     "gba_token_list_create": (ctypes.c_int, [ctypes.c_int64, ctypes.c_int32, ctypes.POINTER(_P)]),
     "gba_fetch_token": (ctypes.c_int, [_P, ctypes.POINTER(ctypes.c_int64)]),
@@ -293,17 +295,18 @@ class GBA:
         w, s0, s1, v = _P(), _P(), _P(), _P()
         check(self.L.gba_get_table(self.h, t, ctypes.byref(w), ctypes.byref(s0),
                                    ctypes.byref(s1), ctypes.byref(v)), self.h)
-        n = self.rows[t] * self.dims[t]
+        rows = self.capacity(t)
+        n = rows * self.dims[t]
         torch = self.torch
         self.sync()
         out = []
         for p, cnt, dt in ((w, n, torch.float32), (s0, n, torch.float32), (s1, n, torch.float32),
-                           (v, self.rows[t], torch.int32)):
+                           (v, rows, torch.int32)):
             out.append(None if not p.value else _copy_device(p.value, cnt, dt))
-        out[0] = out[0].view(self.rows[t], self.dims[t])
-        out[1] = out[1].view(self.rows[t], self.dims[t])
+        out[0] = out[0].view(rows, self.dims[t])
+        out[1] = out[1].view(rows, self.dims[t])
         if out[2] is not None:
-            out[2] = out[2].view(self.rows[t], self.dims[t])
+            out[2] = out[2].view(rows, self.dims[t])
         return out
 
     def table_rows(self, t, rows):
@@ -314,14 +317,15 @@ class GBA:
         self.sync()
         torch = self.torch
         d = self.dims[t]
+        cap = self.capacity(t)
         idx = torch.as_tensor(rows, dtype=torch.int64, device="cuda")
         res = []
         for p in (w, s0, s1):
             if not p.value:
                 res.append(None)
                 continue
-            res.append(_gather_rows(p.value, self.rows[t], d, idx))
-        res.append(_gather_rows(v.value, self.rows[t], 1, idx, torch.int32).view(-1))
+            res.append(_gather_rows(p.value, cap, d, idx))
+        res.append(_gather_rows(v.value, cap, 1, idx, torch.int32).view(-1))
         return res
 
     def dense(self):
@@ -346,6 +350,22 @@ class GBA:
         check(self.L.gba_pull(self.h, int(t), ids.data_ptr() if ids.numel() else None,
                               ids.numel(), out.data_ptr() if ids.numel() else None),
               self.h, "gba_pull")
+        return out
+
+    def capacity(self, t):
+        """Rows the arrays of table t hold now (slots of a HASH table)."""
+        r = ctypes.c_int64()
+        check(self.L.gba_table_capacity(self.h, int(t), ctypes.byref(r)), self.h)
+        return int(r.value)
+
+    def lookup(self, t, ids):
+        """Slots of the device int64 tensor ids in HASH table t (-1: absent)."""
+        torch = self.torch
+        ids = ids.contiguous()
+        out = torch.empty(ids.numel(), dtype=torch.int64, device=ids.device)
+        if ids.numel():
+            check(self.L.gba_lookup_rows(self.h, int(t), ids.data_ptr(), ids.numel(),
+                                         out.data_ptr()), self.h, "gba_lookup_rows")
         return out
 
     def set_eager_dense(self, on=True):

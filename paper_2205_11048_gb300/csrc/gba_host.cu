@@ -47,7 +47,7 @@ struct Arena {  // contiguous-allocation ring over [0, cap) with virtual offsets
 };
 
 struct TableState {
-  gba_table_desc desc;
+  gba_table_desc desc;  // for a HASH table, rows is the current number of slots
   float* w = nullptr;
   float* s0 = nullptr;
   float* s1 = nullptr;
@@ -55,6 +55,11 @@ struct TableState {
   uint32_t key_base = 0;
   double bpow1 = 1.0, bpow2 = 1.0;  // beta^t of Adam, as successive products
   Arena arena;
+  // HASH tables: slot keys, inserted-id counter, and a bound on the ids
+  // inserted so far (exact at the last read plus every occurrence since)
+  unsigned long long* keys = nullptr;
+  unsigned long long* count = nullptr;
+  int64_t id_bound = 0;
 };
 
 struct Msg {
@@ -115,6 +120,9 @@ struct gba_handle {
 
   TableInfo* d_tinfo = nullptr;
   std::vector<TableInfo> h_tinfo;
+  HashInfo* d_hinfo = nullptr;
+  std::vector<HashInfo> h_hinfo;
+  uint64_t seed_table = 0;
 
   size_t meta_bytes = 0;
   char* d_meta[SLOTS] = {};
@@ -286,9 +294,12 @@ void free_all(gba_handle* h) {
     cudaFree(t.s0);
     cudaFree(t.s1);
     cudaFree(t.ver);
+    cudaFree(t.keys);
+    cudaFree(t.count);
     cudaFree(t.arena.ids);
     cudaFree(t.arena.rows);
   }
+  cudaFree(h->d_hinfo);
   cudaFree(h->dw);
   cudaFree(h->ds0);
   cudaFree(h->ds1);
@@ -377,6 +388,105 @@ gba_status poll_device_error(gba_handle* h, bool force_sync) {
     h->fail_code = set_err(h, GBA_E_CUDA, "device consistency check failed");
   }
   return h->fail_code;
+}
+
+HashInfo hash_info(const gba_handle* h, int t) {
+  const TableState& ts = h->tables[t];
+  HashInfo hi{};
+  hi.keys = ts.keys;
+  hi.mask = (uint64_t)ts.desc.rows - 1;
+  hi.w = ts.w;
+  hi.s0 = ts.s0;
+  hi.s1 = ts.s1;
+  hi.ver = ts.ver;
+  hi.count = ts.count;
+  hi.seed = h->seed;
+  hi.tag = ((uint64_t)(uint32_t)t + 1u) << 48;
+  hi.d = ts.desc.dim;
+  hi.kind = ts.desc.opt.kind;
+  hi.init_acc = ts.desc.opt.adagrad_init_acc;
+  return hi;
+}
+
+// Key bases (tables in order), key bits and sort passes from the tables' rows,
+// and the device copies of the table and hash descriptions.
+gba_status layout_keys(gba_handle* h) {
+  uint64_t base = 0;
+  for (int t = 0; t < h->T; ++t) {
+    TableState& ts = h->tables[t];
+    ts.key_base = (uint32_t)base;
+    h->h_tinfo[t] = TableInfo{ts.desc.rows, (uint32_t)base, ts.desc.id_mode,
+                              ~0ull / (uint64_t)ts.desc.rows};
+    h->h_hinfo[t] = ts.desc.id_mode == GBA_ID_HASH ? hash_info(h, t) : HashInfo{};
+    base += (uint64_t)ts.desc.rows;
+  }
+  if (base >= 0xFFFFFFFFull) return set_err(h, GBA_E_ARG, "tables hold 2^32 - 1 rows or more");
+  const uint64_t kmax = base > 0 ? base - 1 : 0;
+  uint32_t bits = 1;
+  while (bits < 32 && (kmax >> bits) != 0) ++bits;
+  h->total_keys_bits = bits;
+  h->passes = (int)((bits + 7) / 8);
+  if (h->T > 0) {
+    GBA_CUDA(h, cudaMemcpy(h->d_tinfo, h->h_tinfo.data(), h->T * sizeof(TableInfo),
+                           cudaMemcpyHostToDevice));
+    GBA_CUDA(h, cudaMemcpy(h->d_hinfo, h->h_hinfo.data(), h->T * sizeof(HashInfo),
+                           cudaMemcpyHostToDevice));
+  }
+  return GBA_OK;
+}
+
+// A HASH table's arrays for `slots` slots (keys cleared; rows are initialised
+// when their id is inserted).
+gba_status alloc_hash_arrays(gba_handle* h, TableState& ts, uint64_t slots) {
+  const size_t n = (size_t)slots * ts.desc.dim;
+  GBA_CUDA(h, cudaMalloc(&ts.w, n * 4));
+  GBA_CUDA(h, cudaMalloc(&ts.s0, n * 4));
+  if (ts.desc.opt.kind == GBA_ADAM) GBA_CUDA(h, cudaMalloc(&ts.s1, n * 4));
+  GBA_CUDA(h, cudaMalloc(&ts.ver, (size_t)slots * 4));
+  GBA_CUDA(h, cudaMalloc(&ts.keys, (size_t)slots * 8));
+  launch_hash_clear(ts.keys, slots, h->stream);
+  GBA_CUDA(h, cudaGetLastError());
+  return GBA_OK;
+}
+
+// Keeps every HASH table at most half full for the step about to run: the
+// bound on its ids grows by the step's occurrences; when it passes half the
+// slots the exact count is read, and if that is still too many the table
+// doubles until it is not, every id moving to its slot in the larger table.
+gba_status grow_hash_tables(gba_handle* h, const std::vector<int64_t>& nbase) {
+  bool changed = false;
+  for (int t = 0; t < h->T; ++t) {
+    TableState& ts = h->tables[t];
+    if (ts.desc.id_mode != GBA_ID_HASH) continue;
+    const int64_t Nt = nbase[t + 1] - nbase[t];
+    ts.id_bound += Nt;
+    if (ts.id_bound <= ts.desc.rows / 2) continue;
+    GBA_CUDA(h, sync_all(h));
+    unsigned long long have = 0;
+    GBA_CUDA(h, cudaMemcpy(&have, ts.count, 8, cudaMemcpyDeviceToHost));
+    ts.id_bound = (int64_t)have + Nt;
+    if (ts.id_bound <= ts.desc.rows / 2) continue;
+    uint64_t slots = (uint64_t)ts.desc.rows;
+    while ((int64_t)(slots / 2) < ts.id_bound) slots *= 2;
+    const HashInfo from = hash_info(h, t);
+    TableState old = ts;
+    ts.w = ts.s0 = ts.s1 = nullptr;
+    ts.ver = nullptr;
+    ts.keys = nullptr;
+    gba_status st = alloc_hash_arrays(h, ts, slots);
+    if (st != GBA_OK) return st;
+    ts.desc.rows = (int64_t)slots;
+    launch_hash_rehash(from, hash_info(h, t), h->stream);
+    GBA_CUDA(h, cudaGetLastError());
+    GBA_CUDA(h, cudaStreamSynchronize(h->stream));
+    cudaFree(old.w);
+    cudaFree(old.s0);
+    cudaFree(old.s1);
+    cudaFree(old.ver);
+    cudaFree(old.keys);
+    changed = true;
+  }
+  return changed ? layout_keys(h) : GBA_OK;
 }
 
 gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
@@ -599,10 +709,18 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   for (int t = 0; t < n_tables; ++t) {
     const gba_table_desc& d = tables[t];
     if (d.rows < 1 || d.dim < 1 || d.dim > MAX_DIM) return GBA_E_ARG;
-    if (d.id_mode != GBA_ID_DIRECT && d.id_mode != GBA_ID_MODULO) return GBA_E_ARG;
+    if (d.id_mode != GBA_ID_DIRECT && d.id_mode != GBA_ID_MODULO && d.id_mode != GBA_ID_HASH)
+      return GBA_E_ARG;
+    if (d.id_mode == GBA_ID_HASH && d.rows > (1ll << 30)) return GBA_E_ARG;
     if (d.max_ids_per_msg < 0 || d.max_ids_per_msg > MAX_STEP_OCC) return GBA_E_ARG;
     if (validate_opt(d.opt) != GBA_OK) return GBA_E_ARG;
-    total_rows += (uint64_t)d.rows;
+    uint64_t r = (uint64_t)d.rows;
+    if (d.id_mode == GBA_ID_HASH) {  // a power of two of slots, at least 1024
+      uint64_t slots = 1024;
+      while (slots < r) slots *= 2;
+      r = slots;
+    }
+    total_rows += r;
   }
   if (total_rows >= 0xFFFFFFFFull) return GBA_E_ARG;  // keys are 32-bit, one value reserved
   if (dense_size > 0 && validate_opt(*dense_opt) != GBA_OK) return GBA_E_ARG;
@@ -659,25 +777,19 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
         return fail(GBA_E_CUDA);
   if (configure_dense() != cudaSuccess) return fail(GBA_E_CUDA);
 
-  // key space: tables in order
-  uint32_t base = 0;
+  // tables (a HASH table starts with a power of two of slots)
   h->tables.resize(n_tables);
   h->h_tinfo.resize(n_tables);
+  h->h_hinfo.resize(n_tables);
   for (int t = 0; t < n_tables; ++t) {
     TableState& ts = h->tables[t];
     ts.desc = tables[t];
-    ts.key_base = base;
-    h->h_tinfo[t] = TableInfo{tables[t].rows, base, tables[t].id_mode,
-                              ~0ull / (uint64_t)tables[t].rows};
-    base += (uint32_t)tables[t].rows;
+    if (ts.desc.id_mode == GBA_ID_HASH) {
+      int64_t slots = 1024;
+      while (slots < ts.desc.rows) slots *= 2;
+      ts.desc.rows = slots;
+    }
     h->d_max = std::max(h->d_max, (int)tables[t].dim);
-  }
-  {
-    uint64_t kmax = total_rows > 0 ? total_rows - 1 : 0;
-    uint32_t bits = 1;
-    while (bits < 32 && (kmax >> bits) != 0) ++bits;
-    h->total_keys_bits = bits;
-    h->passes = (int)((bits + 7) / 8);
   }
 
   auto dev_alloc = [&](void** p, size_t bytes) -> bool {
@@ -686,6 +798,12 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   };
   for (int t = 0; t < n_tables; ++t) {
     TableState& ts = h->tables[t];
+    if (ts.desc.id_mode == GBA_ID_HASH) {
+      if (alloc_hash_arrays(h, ts, (uint64_t)ts.desc.rows) != GBA_OK ||
+          !dev_alloc((void**)&ts.count, 8) || cudaMemset(ts.count, 0, 8) != cudaSuccess)
+        return fail(GBA_E_OOM);
+      continue;
+    }
     const size_t n = (size_t)ts.desc.rows * ts.desc.dim;
     if (!dev_alloc((void**)&ts.w, n * 4) || !dev_alloc((void**)&ts.s0, n * 4) ||
         (ts.desc.opt.kind == GBA_ADAM && !dev_alloc((void**)&ts.s1, n * 4)) ||
@@ -697,12 +815,13 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
         (h->dense_opt.kind == GBA_ADAM && !dev_alloc((void**)&h->ds1, h->D_pad * 4)))
       return fail(GBA_E_OOM);
   }
+  h->seed = init_seed;
   if (n_tables > 0) {
-    if (!dev_alloc((void**)&h->d_tinfo, n_tables * sizeof(TableInfo))) return fail(GBA_E_OOM);
-    if (cudaMemcpy(h->d_tinfo, h->h_tinfo.data(), n_tables * sizeof(TableInfo),
-                   cudaMemcpyHostToDevice) != cudaSuccess)
-      return fail(GBA_E_CUDA);
+    if (!dev_alloc((void**)&h->d_tinfo, n_tables * sizeof(TableInfo)) ||
+        !dev_alloc((void**)&h->d_hinfo, n_tables * sizeof(HashInfo)))
+      return fail(GBA_E_OOM);
   }
+  if (layout_keys(h) != GBA_OK) return fail(GBA_E_CUDA);
   // step descriptor buffers
   {
     const size_t M = (size_t)max_buffered_msgs, T = (size_t)n_tables;
@@ -775,6 +894,7 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   // initial values (R11 of the design notes: counter-based hash of (seed, array, element))
   for (int t = 0; t < n_tables; ++t) {
     TableState& ts = h->tables[t];
+    if (ts.desc.id_mode == GBA_ID_HASH) continue;  // rows start when their id arrives
     Timed tm(h, GBA_K_INIT, h->stream);
     launch_init_table(ts.w, ts.s0, ts.s1, ts.ver, ts.desc.rows, ts.desc.dim, ts.desc.opt.kind,
                       ts.desc.opt.adagrad_init_acc, init_seed, ((uint64_t)(uint32_t)t + 1u) << 48,
@@ -831,7 +951,8 @@ int32_t gba_try_apply(gba_handle* h) {
   if (N > MAX_STEP_OCC) return set_err(h, GBA_E_ARG, "more than 2^30-1 ids in one global step");
   cudaSetDevice(h->device);
   {
-    gba_status s = ensure_step_capacity(h, N);
+    gba_status s = grow_hash_tables(h, nbase);
+    if (s == GBA_OK) s = ensure_step_capacity(h, N);
     if (s != GBA_OK) return s;
   }
 
@@ -911,6 +1032,7 @@ int32_t gba_try_apply(gba_handle* h) {
   a.rows_ptr = (const float* const*)(dmeta + o_rows);
   a.nbase = (const int64_t*)(dmeta + o_nbase);
   a.tinfo = h->d_tinfo;
+  a.hinfo = h->d_hinfo;
 
   // ---- K1: message weights (Eq. (1)); clears the per-step scratch
   {
@@ -1154,8 +1276,8 @@ gba_status gba_pull(gba_handle* h, int32_t t, const int64_t* ids, int64_t n, flo
   const TableState& ts = h->tables[t];
   ErrSink sink = h->sink;
   sink.step = h->d_err;  // no step of its own: the handle's word takes both roles
-  launch_pull_rows(ts.w, ts.desc.rows, ts.desc.dim, ts.desc.id_mode, h->h_tinfo[t].mod_magic, ids,
-                   n, out, sink, h->num_sms, h->stream);
+  launch_pull_rows(ts.w, ts.desc.rows, ts.desc.dim, ts.desc.id_mode, h->h_tinfo[t].mod_magic,
+                   h->d_hinfo + t, ids, n, out, sink, h->num_sms, h->stream);
   GBA_CUDA(h, cudaGetLastError());
   return GBA_OK;
 }
@@ -1175,6 +1297,24 @@ gba_status gba_set_eager_dense(gba_handle* h, int32_t on) {
       GBA_CUDA(h, cudaEventCreateWithFlags(&h->acc_ev[i], cudaEventDisableTiming));
   }
   h->eager = on != 0;
+  return GBA_OK;
+}
+
+gba_status gba_table_capacity(gba_handle* h, int32_t t, int64_t* rows) {
+  if (!h || t < 0 || t >= h->T || !rows) return GBA_E_ARG;
+  *rows = h->tables[t].desc.rows;
+  return GBA_OK;
+}
+
+gba_status gba_lookup_rows(gba_handle* h, int32_t t, const int64_t* ids, int64_t n,
+                           int64_t* rows_out) {
+  if (!h || t < 0 || t >= h->T || n < 0) return GBA_E_ARG;
+  if (h->tables[t].desc.id_mode != GBA_ID_HASH) return set_err(h, GBA_E_ARG, "not a HASH table");
+  if (n > 0 && (!ids || !rows_out)) return set_err(h, GBA_E_ARG, "NULL ids or rows_out");
+  cudaSetDevice(h->device);
+  join_steps(h);
+  launch_hash_lookup(h->d_hinfo + t, ids, n, rows_out, h->stream);
+  GBA_CUDA(h, cudaGetLastError());
   return GBA_OK;
 }
 
@@ -1220,10 +1360,16 @@ gba_status gba_debug_segments(gba_handle* h, int64_t cap, int32_t* table, int64_
     std::vector<uint4> rr((size_t)U[t] + 1);
     GBA_CUDA(h, cudaMemcpy(rr.data(), h->d_rr + h->last_nbase[t] + t, rr.size() * sizeof(uint4),
                            cudaMemcpyDeviceToHost));
+    std::vector<unsigned long long> keys;  // HASH tables report the id of each slot
+    if (h->tables[t].desc.id_mode == GBA_ID_HASH) {
+      keys.resize((size_t)h->tables[t].desc.rows);
+      GBA_CUDA(h, cudaMemcpy(keys.data(), h->tables[t].keys, keys.size() * 8,
+                             cudaMemcpyDeviceToHost));
+    }
     for (uint32_t u = 0; u < U[t]; ++u, ++u_all) {
       if (u_all >= cap) continue;
       if (table) table[u_all] = t;
-      if (row) row[u_all] = (int64_t)rr[u].x;
+      if (row) row[u_all] = keys.empty() ? (int64_t)rr[u].x : (int64_t)keys[rr[u].x];
       if (count) count[u_all] = (int64_t)(rr[u + 1].z - rr[u].z);
       if (kept) kept[u_all] = (int64_t)(rr[u + 1].y - rr[u].y);
     }

@@ -106,6 +106,89 @@ __device__ __forceinline__ uint64_t mod_u64(uint64_t x, uint64_t V, uint64_t m) 
   return r;
 }
 
+// ---- counter-based initial values (shared by table init and hash inserts) ---
+// SplitMix64 (Steele, Lea, Flood 2014): output for state x.
+__device__ __forceinline__ uint64_t splitmix64(uint64_t x) {
+  uint64_t z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+// Weight of element e of an array: top 24 bits of the hash, centred, times
+// 2^-27 (an exact float in [-1/16, 1/16)).
+__device__ __forceinline__ float init_weight(uint64_t seed, uint64_t tag, uint64_t e) {
+  const uint64_t h = splitmix64(seed ^ tag ^ e);
+  const int32_t top = (int32_t)(h >> 40) - 8388608;
+  return (float)top * 0x1p-27f;
+}
+
+// ---- expandable hash tables of 64-bit ids (id_mode HASH) --------------------
+// Open addressing with linear probing over a power-of-two number of slots; the
+// row of an id is the slot it occupies, so the embedding arrays are indexed by
+// slot.  A new id is inserted by compare-and-swap on its slot's key and its
+// row is initialised from the id (element e = id * d + j of the table's
+// counter-based stream), so every id starts from the same values whichever
+// slot it lands in.
+constexpr unsigned long long HASH_EMPTY = 0x8000000000000000ull;  // INT64_MIN: not a valid id
+struct HashInfo {
+  unsigned long long* keys;  // [slots] id per slot, HASH_EMPTY when free
+  uint64_t mask;             // slots - 1
+  float* w;
+  float* s0;
+  float* s1;
+  int32_t* ver;
+  unsigned long long* count;  // ids inserted so far
+  uint64_t seed, tag;
+  int32_t d, kind;
+  float init_acc;
+  int32_t pad;
+};
+
+__device__ __forceinline__ void hash_init_row(const HashInfo& hi, uint64_t slot, int64_t id) {
+  const float a0 = hi.kind == 0 ? hi.init_acc : 0.f;
+  for (int j = 0; j < hi.d; ++j) {
+    const size_t e = (size_t)slot * hi.d + j;
+    hi.w[e] = init_weight(hi.seed, hi.tag, (uint64_t)id * (uint64_t)hi.d + (uint64_t)j);
+    hi.s0[e] = a0;
+    if (hi.kind == 1) hi.s1[e] = 0.f;
+  }
+  hi.ver[slot] = 0;
+}
+
+// The slot of id, inserting it when absent; returns mask + 1 when the table
+// is full (cannot happen while the host keeps it at most half full).
+__device__ __forceinline__ uint64_t hash_find_or_insert(const HashInfo& hi, int64_t id) {
+  const unsigned long long key = (unsigned long long)id;
+  uint64_t slot = splitmix64(key) & hi.mask;
+  for (uint64_t probe = 0; probe <= hi.mask; ++probe, slot = (slot + 1) & hi.mask) {
+    const unsigned long long k = *(volatile unsigned long long*)(hi.keys + slot);
+    if (k == key) return slot;
+    if (k == HASH_EMPTY) {
+      const unsigned long long old = atomicCAS(hi.keys + slot, HASH_EMPTY, key);
+      if (old == HASH_EMPTY) {
+        hash_init_row(hi, slot, id);
+        atomicAdd(hi.count, 1ull);
+        return slot;
+      }
+      if (old == key) return slot;
+    }
+  }
+  return hi.mask + 1;
+}
+
+// The slot of id, or mask + 1 when it is absent.
+__device__ __forceinline__ uint64_t hash_find(const HashInfo& hi, int64_t id) {
+  const unsigned long long key = (unsigned long long)id;
+  uint64_t slot = splitmix64(key) & hi.mask;
+  for (uint64_t probe = 0; probe <= hi.mask; ++probe, slot = (slot + 1) & hi.mask) {
+    const unsigned long long k = hi.keys[slot];
+    if (k == key) return slot;
+    if (k == HASH_EMPTY) break;
+  }
+  return hi.mask + 1;
+}
+
 // ---- optimizer parameters of one parameter group for one step ---------------
 struct OptStep {
   int32_t kind;  // 0 Adagrad, 1 Adam
@@ -186,6 +269,7 @@ struct StepArgs {
   const float* const* rows_ptr;   // [T][M]
   const int64_t* nbase;           // [T+1] first global occurrence of each table
   const TableInfo* tinfo;         // [T]
+  const HashInfo* hinfo;          // [T] (tables with id_mode HASH)
 };
 
 // Per-step device scratch that K1 clears at the start of a step.
@@ -358,8 +442,15 @@ int launch_wait_selftest(int64_t limit_ns, cudaStream_t s, uint32_t* d_word, uin
 
 // Rows of one table for n ids (pull responding), into out[n][d].
 void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, uint64_t mod_magic,
-                      const int64_t* ids, int64_t n, float* out, ErrSink err, int num_sms,
-                      cudaStream_t s);
+                      const HashInfo* hinfo, const int64_t* ids, int64_t n, float* out,
+                      ErrSink err, int num_sms, cudaStream_t s);
+
+// Hash tables: fill keys with HASH_EMPTY; move every id of one table into a
+// larger one (keys, rows and tags); slots of ids (mask + 1 when absent).
+void launch_hash_clear(unsigned long long* keys, uint64_t slots, cudaStream_t s);
+void launch_hash_rehash(HashInfo from, HashInfo to, cudaStream_t s);
+void launch_hash_lookup(const HashInfo* hinfo, const int64_t* ids, int64_t n, int64_t* slots,
+                        cudaStream_t s);
 
 // Compute capability (major * 10 + minor) of the device code the library's
 // kernels were loaded from on the current device, or -1.

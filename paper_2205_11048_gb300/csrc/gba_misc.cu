@@ -5,21 +5,6 @@ namespace gba {
 
 namespace {
 
-// SplitMix64 (Steele, Lea, Flood 2014): output for state x.
-__device__ __forceinline__ uint64_t splitmix64(uint64_t x) {
-  uint64_t z = x + 0x9E3779B97F4A7C15ull;
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-
-// Weight of element e: top 24 bits of the hash, centred, times 2^-27 (exact).
-__device__ __forceinline__ float init_weight(uint64_t seed, uint64_t tag, uint64_t e) {
-  const uint64_t h = splitmix64(seed ^ tag ^ e);
-  const int32_t top = (int32_t)(h >> 40) - 8388608;
-  return (float)top * 0x1p-27f;
-}
-
 __global__ void k_init_params(float* __restrict__ w, float* __restrict__ s0,
                               float* __restrict__ s1, int64_t n, int32_t kind, float init_acc,
                               uint64_t seed, uint64_t tag) {
@@ -81,6 +66,57 @@ int launch_wait_selftest(int64_t limit_ns, cudaStream_t s, uint32_t* d_word, uin
     return -1;
   if (cudaStreamSynchronize(s) != cudaSuccess) return -1;
   return 0;
+}
+
+namespace {
+
+__global__ void k_hash_clear(unsigned long long* keys, uint64_t slots) {
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < slots; i += stride)
+    keys[i] = HASH_EMPTY;
+}
+
+// Every occupied slot of `from` moves to its slot in `to` (no id repeats, so
+// the insert never meets its own id), with its row, state and tag.
+__global__ void k_hash_rehash(HashInfo from, HashInfo to) {
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i <= from.mask; i += stride) {
+    const unsigned long long key = from.keys[i];
+    if (key == HASH_EMPTY) continue;
+    uint64_t slot = splitmix64(key) & to.mask;
+    for (uint64_t probe = 0; probe <= to.mask; ++probe, slot = (slot + 1) & to.mask)
+      if (atomicCAS(to.keys + slot, HASH_EMPTY, key) == HASH_EMPTY) break;
+    for (int j = 0; j < from.d; ++j) {
+      to.w[slot * from.d + j] = from.w[i * from.d + j];
+      to.s0[slot * from.d + j] = from.s0[i * from.d + j];
+      if (from.kind == 1) to.s1[slot * from.d + j] = from.s1[i * from.d + j];
+    }
+    to.ver[slot] = from.ver[i];
+  }
+}
+
+__global__ void k_hash_lookup(const HashInfo* hinfo, const int64_t* ids, int64_t n, int64_t* slots) {
+  const HashInfo hi = *hinfo;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const uint64_t s = hash_find(hi, ids[i]);
+    slots[i] = s > hi.mask ? -1 : (int64_t)s;
+  }
+}
+
+}  // namespace
+
+void launch_hash_clear(unsigned long long* keys, uint64_t slots, cudaStream_t s) {
+  k_hash_clear<<<grid_for((int64_t)slots), 256, 0, s>>>(keys, slots);
+}
+
+void launch_hash_rehash(HashInfo from, HashInfo to, cudaStream_t s) {
+  k_hash_rehash<<<grid_for((int64_t)from.mask + 1), 256, 0, s>>>(from, to);
+}
+
+void launch_hash_lookup(const HashInfo* hinfo, const int64_t* ids, int64_t n, int64_t* slots,
+                        cudaStream_t s) {
+  if (n > 0) k_hash_lookup<<<grid_for(n), 256, 0, s>>>(hinfo, ids, n, slots);
 }
 
 int kernel_binary_version() {

@@ -18,8 +18,8 @@ constexpr int PULL_THREADS = 256;
 template <bool VEC>
 __global__ void __launch_bounds__(PULL_THREADS)
     k_pull_rows(const float* __restrict__ w, int64_t V, int d, int id_mode, uint64_t mod_magic,
-                const int64_t* __restrict__ ids, int64_t n, float* __restrict__ out, int lg,
-                ErrSink err) {
+                const HashInfo* hinfo, const int64_t* __restrict__ ids, int64_t n,
+                float* __restrict__ out, int lg, ErrSink err) {
   const int L = 1 << lg;
   const int lane = threadIdx.x & 31;
   const int l = lane & (L - 1);
@@ -29,15 +29,25 @@ __global__ void __launch_bounds__(PULL_THREADS)
     const int64_t id = __ldg(ids + i);
     bool ok = true;
     uint64_t row;
+    bool fresh = false;  // HASH: an id never seen gets its initial values
     if (id_mode == 0) {
       ok = id >= 0 && id < V;
       row = ok ? (uint64_t)id : 0ull;
-    } else {
+    } else if (id_mode == 1) {
       row = mod_u64((uint64_t)id, (uint64_t)V, mod_magic);
+    } else {
+      row = hash_find(*hinfo, id);
+      fresh = row > hinfo->mask;
+      if (fresh) row = 0;
     }
     if (!ok && l == 0) raise_error(err, ERR_ID_RANGE);
     const float* src = w + row * (uint64_t)d;
     float* dst = out + (uint64_t)i * (uint64_t)d;
+    if (fresh) {
+      for (int q = l; q < d; q += L)
+        dst[q] = init_weight(hinfo->seed, hinfo->tag, (uint64_t)id * (uint64_t)d + (uint64_t)q);
+      continue;
+    }
     if (VEC) {
       const int C = d >> 2;
       for (int q = l; q < C; q += L) {
@@ -54,8 +64,8 @@ __global__ void __launch_bounds__(PULL_THREADS)
 }  // namespace
 
 void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, uint64_t mod_magic,
-                      const int64_t* ids, int64_t n, float* out, ErrSink err, int num_sms,
-                      cudaStream_t s) {
+                      const HashInfo* hinfo, const int64_t* ids, int64_t n, float* out,
+                      ErrSink err, int num_sms, cudaStream_t s) {
   if (n <= 0) return;
   const bool vec = (d & 3) == 0 && ((uintptr_t)out & 15u) == 0;
   const int pieces = vec ? d / 4 : d;
@@ -66,10 +76,10 @@ void launch_pull_rows(const float* w, int64_t V, int d, int id_mode, uint64_t mo
   const int64_t cap = (int64_t)num_sms * 8;
   if (grid > cap) grid = cap;
   if (vec)
-    k_pull_rows<true><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, mod_magic, ids, n, out, lg, err);
+    k_pull_rows<true><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, mod_magic, hinfo, ids, n, out, lg, err);
   else
-    k_pull_rows<false><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, mod_magic, ids, n,
-                                                               out, lg, err);
+    k_pull_rows<false><<<(unsigned)grid, PULL_THREADS, 0, s>>>(w, V, d, id_mode, mod_magic, hinfo,
+                                                               ids, n, out, lg, err);
 }
 
 }  // namespace gba

@@ -91,8 +91,19 @@ __device__ __forceinline__ uint32_t occurrence_key(const StepArgs& a, const uint
     } else {
       row = (uint64_t)id;
     }
-  } else {
+  } else if (ti.id_mode == 1) {
     row = mod_u64((uint64_t)id, (uint64_t)ti.V, ti.mod_magic);
+  } else {  // HASH: the id's slot, inserted on first sight
+    if ((unsigned long long)id == HASH_EMPTY) {
+      raise_error(err, ERR_ID_RANGE);
+      row = 0;
+    } else {
+      row = hash_find_or_insert(a.hinfo[t], id);
+      if (row > a.hinfo[t].mask) {
+        raise_error(err, ERR_INTERNAL);
+        row = 0;
+      }
+    }
   }
   return ti.key_base + (uint32_t)row;
 }

@@ -28,6 +28,7 @@ ADAGRAD = 0
 ADAM = 1
 DIRECT = 0
 MODULO = 1
+HASH = 2
 
 
 @dataclass(frozen=True)
@@ -47,7 +48,7 @@ class TableCfg:
     fields: int               # feature fields that look up this table
     ids_per_field: float = 0  # 0: one id per sample and field; >0: Poisson mean
     zipf: float = 1.05        # exponent of the bounded Zipf law over ranks 1..rows
-    id_mode: int = DIRECT     # DIRECT: id is the row; MODULO: 64-bit hashed id
+    id_mode: int = DIRECT     # DIRECT: id is the row; MODULO / HASH: 64-bit hashed id
     opt: OptCfg = field(default_factory=OptCfg)
 
 

@@ -61,8 +61,10 @@ def rel_err(a: np.ndarray, b: np.ndarray) -> float:
 
 
 def rows_of(cfg, t, ids_np):
+    """The oracle's row of each id: the id itself (DIRECT, and HASH tables,
+    where every distinct id is a row), or its unsigned residue (MODULO)."""
     tb = cfg.tables[t]
-    if tb.id_mode == W.DIRECT:
+    if tb.id_mode in (W.DIRECT, W.HASH):
         return ids_np.astype(np.int64)
     return (ids_np.view(np.uint64) % np.uint64(tb.rows)).astype(np.int64)
 

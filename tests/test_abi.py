@@ -56,7 +56,8 @@ def _create(L, tables, D=8, G=4, max_buf=4, st=None, dense_opt=None):
 
 @pytest.mark.parametrize("bad", [
     dict(tables=[_table(rows=0)]), dict(tables=[_table(dim=0)]), dict(tables=[_table(dim=257)]),
-    dict(tables=[_table(mode=2)]), dict(tables=[_table(mx=-1)]),
+    dict(tables=[_table(mode=3)]), dict(tables=[_table(mx=-1)]),
+    dict(tables=[_table(mode=2, rows=2**30 + 1)]),
     dict(tables=[_table(kind=5)]), dict(tables=[_table(init=0.0)]),
     dict(tables=[_table(rows=2**31), _table(rows=2**31)]),
     dict(tables=[_table()], G=0), dict(tables=[_table()], max_buf=0),

@@ -576,3 +576,76 @@ def test_eager_dense_refusals_and_capacity():
     assert g.try_apply() == 0
     g.sync()
     g.close()
+
+
+def test_hash_table_grows_and_matches_the_oracle():
+    """An expandable hash table of 64-bit ids (every distinct id its own row)
+    next to a DIRECT table: it starts at 1024 slots and doubles several times
+    as new ids arrive; dedup output, state, tags and pulls (of stored and of
+    never-seen ids) match the oracle, which keys rows by id."""
+    rng = np.random.default_rng(23)
+    ranks = 30_000
+    salt = 0x5DEECE66D
+    tcs = (W.TableCfg(1000, 16, 1, 0, 1.1, W.HASH, W.OptCfg(W.ADAGRAD, 0.01)),
+           W.TableCfg(300, 8, 1, 0, 1.1, W.DIRECT, W.OptCfg(W.ADAM, 0.001)))
+    cfg = W.WorkloadCfg("hash", M=4, B=1, tables=tcs, D=77, dense_opt=W.OptCfg(W.ADAM, 0.001),
+                        stale=W.StaleCfg("fresh"), iota=2, seed=8)
+    steps = []
+    for k in range(8):
+        batch = []
+        for m in range(4):
+            r = torch.as_tensor(rng.zipf(1.2, 2000) % ranks, dtype=torch.int64)
+            ids0 = W.hash64(r ^ salt)
+            ids1 = rng.integers(0, 300, 50)
+            batch.append(msg(max(0, k - int(rng.integers(0, 4))), [ids0.numpy(), ids1], [16, 8], 77))
+        steps.append(batch)
+    all_ids = np.unique(np.concatenate([m["ids"][0].cpu().numpy() for b in steps for m in b]))
+    unseen = W.hash64(torch.arange(ranks, ranks + 40, dtype=torch.int64) ^ salt).numpy()
+    track0 = np.unique(np.concatenate([all_ids, unseen]))
+    tables = [(1000, 16, W.HASH, 8192, H.opt_desc(tcs[0].opt)),
+              (300, 8, W.DIRECT, 8192, H.opt_desc(tcs[1].opt))]
+    g = B.GBA(tables, 77, H.opt_desc(cfg.dense_opt), 4, 16, seed=cfg.seed, iota=2)
+    g.set_debug(True)
+    assert g.capacity(0) == 1024
+    orc = H.make_oracle(cfg, track_rows=[track0, None])
+    for batch in steps:
+        for m in batch:
+            g.push(m["token"], m["ids"], m["rows"], m["dense"], 1)
+            orc.push(H.to_oracle(m))
+        assert g.try_apply() == 1 and orc.try_apply() == 1
+        # dedup output: the hash table reports ids; compare as sets ordered by id
+        t_g, r_g, c_g, k_g = g.segments()
+        sel = t_g == 0
+        order = np.argsort(r_g[sel])
+        touched = np.nonzero(orc.last_count[0])[0]
+        assert np.array_equal(r_g[sel][order], track0[touched])
+        assert np.array_equal(c_g[sel][order], orc.last_count[0][touched])
+        assert np.array_equal(k_g[sel][order], orc.last_kept[0][touched])
+        # state of every tracked id the table holds; ids it does not hold were never pushed
+        slots = g.lookup(0, torch.as_tensor(track0, device="cuda")).cpu().numpy()
+        have = slots >= 0
+        assert np.all(np.isin(track0[have], all_ids))
+        w, s0, _, ver = g.table_rows(0, slots[have])
+        ts = orc.tables[0]
+        assert np.array_equal(ver.cpu().numpy().astype(np.int64), ts.ver[have])
+        assert H.rel_err(w.cpu().numpy(), ts.w.reshape(-1, 16)[have]) <= H.TOL_ONE_STEP
+        assert H.rel_err(s0.cpu().numpy(), ts.s0.reshape(-1, 16)[have]) <= H.TOL_ONE_STEP
+        assert np.all(ts.ver[~have] == 0)
+    assert g.capacity(0) >= 2 * 1024  # the table grew
+    # pulls: stored ids give their rows, never-seen ids their initial values
+    got = g.pull(0, torch.as_tensor(track0, device="cuda")).cpu().numpy()
+    assert H.rel_err(got, orc.tables[0].w.reshape(-1, 16)) <= H.TOL_ONE_STEP
+    unseen_idx = np.searchsorted(track0, unseen)
+    assert np.array_equal(got[unseen_idx], orc.tables[0].w.reshape(-1, 16)[unseen_idx])
+    g.sync()
+    g.close()
+
+
+def test_hash_table_reserved_id_fails_the_step():
+    tables = [(1000, 4, W.HASH, 16, B.opt_desc())]
+    g = B.GBA(tables, 0, None, 1, 4, seed=1)
+    ids = torch.tensor([5, -2**63, 7], dtype=torch.int64, device="cuda")
+    g.push(0, [ids], [torch.zeros(3, 4, device="cuda")], torch.zeros(0, device="cuda"), 1)
+    assert g.L.gba_try_apply(g.h) == 1
+    assert g.L.gba_sync(g.h) == B.GBA_E_ID_RANGE
+    g.close()

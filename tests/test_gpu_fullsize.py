@@ -1,7 +1,13 @@
-"""The five workloads at full size, in the benchmark's launch configuration
-(messages pushed by reference), against the oracle following a sample of rows
-and dense parameters through the same stream (needs a GPU; config 5 holds
-~110 GB of device memory)."""
+"""The five workloads at full size against the oracle (needs a GPU; the
+2e8 x 64 workload holds ~110 GB of device memory).
+
+- sampled: the benchmark's launch configuration (messages pushed by
+  reference, steps overlapping), the oracle following a sample of rows (hot,
+  random, cold) and of dense parameters through the same stream;
+- full tracking: every row and every dense parameter of the 1e7 x 32 and the
+  dense-heavy workloads, with the dedup output (unique rows, per-row message
+  and kept counts) compared bit for bit every step;
+- long: the 1e7 x 32 workload sampled over 100 steps at the many-step bound."""
 import pytest
 import torch
 
@@ -18,12 +24,35 @@ def _built():
     torch.cuda.set_device(0)
 
 
+def _fits(cfg, factor=0.8):
+    free, _ = torch.cuda.mem_get_info()
+    need = sum(t.rows * t.dim * 4 * (2 if t.opt.kind == 0 else 3) for t in cfg.tables)
+    if need > factor * free:
+        pytest.skip(f"needs {need / 1e9:.0f} GB of free device memory")
+
+
 @pytest.mark.parametrize("n", [2, 3, 4, 5])
 def test_full_size_sampled(n):
     cfg = W.config(n)
-    free, total = torch.cuda.mem_get_info()
-    need = sum(t.rows * t.dim * 4 * (2 if t.opt.kind == 0 else 3) for t in cfg.tables)
-    if need > 0.8 * free:
-        pytest.skip(f"needs {need / 1e9:.0f} GB of free device memory")
+    _fits(cfg)
     worst = H.run_fullsize(cfg, steps=3, tol=H.TOL_ONE_STEP)
     print(cfg.name, {k: f"{v:.2e}" for k, v in worst.items()})
+
+
+@pytest.mark.parametrize("n", [2, 4])
+def test_full_size_full_tracking(n):
+    """Every row and dense parameter; dedup output bit-exact each step; one
+    step's bound after the first step, the many-step bound after three."""
+    cfg = W.config(n)
+    _fits(cfg)
+    worst = H.run_parity(cfg, steps=1, tol=H.TOL_ONE_STEP)
+    print(cfg.name, "1 step", {k: f"{v:.2e}" for k, v in worst.items()})
+    worst = H.run_parity(cfg, steps=3, tol=H.TOL_MANY_STEPS, by_ref=True)
+    print(cfg.name, "3 steps", {k: f"{v:.2e}" for k, v in worst.items()})
+
+
+def test_full_size_hundred_steps_sampled():
+    cfg = W.config(2)
+    _fits(cfg)
+    worst = H.run_fullsize(cfg, steps=100, tol=H.TOL_MANY_STEPS)
+    print(cfg.name, "100 steps", {k: f"{v:.2e}" for k, v in worst.items()})
