@@ -34,6 +34,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "global-batch aggregate+apply steps/s; applied grad rows/s; HBM GB/s vs ~8 TB/s peak"
 R_BATCHES = 2
+L2_BYTES = 129e6  # GB300 L2
 
 
 def peaks():
@@ -45,9 +46,22 @@ def peaks():
     return 6800.0, "fallback"
 
 
-def workload_cfg(n):
+def workload_cfg(n, id_mode="as-configured"):
+    """Workload n; id_mode "hash" turns every table into an expandable hash
+    table of 64-bit ids (initial capacity: the next power of two at or above
+    twice its rows)."""
     from paper_2205_11048_gb300 import workload as W
-    return W.config(n)
+    cfg = W.config(n)
+    if id_mode == "hash":
+        def cap(r):
+            c = 1024
+            while c < 2 * r:
+                c *= 2
+            return c
+        cfg = W.replace(cfg, name=cfg.name + "-hash-ids",
+                        tables=tuple(W.replace(t, id_mode=W.HASH, rows=cap(t.rows))
+                                     for t in cfg.tables))
+    return cfg
 
 
 def alg_bytes(cfg, st_delta, steps):
@@ -120,11 +134,21 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def _code_only(text):
+    """C/CUDA source without its comments and blank lines (string literals in
+    these files hold no comment markers)."""
+    import re
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", "", text)
+    return "\n".join(ln.rstrip() for ln in text.splitlines() if ln.strip())
+
+
 def source_sha(files):
+    """Hash of the code (comments excluded) of a kernel class's sources."""
     h = hashlib.sha256()
     for f in files:
-        with open(os.path.join(ROOT, f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, f), encoding="utf-8") as fh:
+            h.update(_code_only(fh.read()).encode())
     return h.hexdigest()[:16]
 
 
@@ -172,6 +196,27 @@ def dist_setup():
     return ws, rank, local
 
 
+def dense_traffic(cfg, per, mode):
+    """Algorithmic dense bytes of one step, split into what the pushes move
+    and what the apply moves.  Buffered (messages pushed by reference): the
+    apply reads every kept message's gradient (4D each) and reads and writes
+    the state.  Eager: a kept push reads its gradient and updates the step's
+    compensated accumulator pair (4D + 8D + 8D; the first kept push of a step
+    only writes it, 4D + 8D), the apply reads the pair (8D) and the state."""
+    D = cfg.D
+    s_opt = 2 if cfg.dense_opt.kind == 0 else 3
+    state = 2 * s_opt * 4 * D
+    m_kept = per["m_kept"]
+    if mode == "eager":
+        push = (12 * D + 20 * D * max(0.0, m_kept - 1)) / max(m_kept, 1e-9) if m_kept else 0.0
+        return {"mode": "eager", "bytes_per_kept_push": push,
+                "bytes_per_apply": 8 * D + state, "bytes_per_step": push * m_kept + 8 * D + state,
+                "buffer_bytes_per_pending_step": 8 * D}
+    return {"mode": "buffered", "bytes_per_kept_push": 0.0,
+            "bytes_per_apply": 4 * D * m_kept + state, "bytes_per_step": 4 * D * m_kept + state,
+            "buffer_bytes_per_message": 4 * D}
+
+
 def config_dict(cfg, ws):
     """The workload description both arms print (the same dict in each)."""
     in_bytes = cfg.M * (sum(cfg.ids_per_msg(t) * (8 + 4 * tb.dim)
@@ -179,8 +224,12 @@ def config_dict(cfg, ws):
     return {"workload": cfg.name, "M": cfg.M, "B": cfg.B, "G": cfg.G,
             "tables": [[t.rows, t.dim] for t in cfg.tables], "dense": cfg.D,
             "iota": cfg.iota, "batches_in_turn": R_BATCHES,
-            "l2": f"inputs larger than L2: each global batch holds {in_bytes / 1e6:.0f} MB of "
-                  f"ids and gradients, {R_BATCHES} distinct batches in turn",
+            "l2": (f"inputs larger than L2: each global batch holds {in_bytes / 1e6:.0f} MB of "
+                   f"ids and gradients, {R_BATCHES} distinct batches in turn"
+                   if in_bytes > L2_BYTES else
+                   f"inputs smaller than L2 (no flush): each global batch holds "
+                   f"{in_bytes / 1e6:.1f} MB of ids and gradients, {R_BATCHES} distinct "
+                   f"batches in turn"),
             "parallelism": f"replicas x{ws}"}
 
 
@@ -239,7 +288,7 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2205_11048_gb300 import workload as W
-    cfg = workload_cfg(args.config)
+    cfg = workload_cfg(args.config, args.id_mode)
     batches = [W.generate_step(cfg, r, "cpu") for r in range(R_BATCHES)]
     sps, sample = oracle_rate(cfg, batches, args.warmup, args.steps)
     line = {"impl": "reference", "metric": METRIC, "value": sps, "unit": "steps/s",
@@ -286,7 +335,7 @@ def run_gba(args):
         __graft_entry__.build()
     L = B.load()
 
-    cfg = workload_cfg(args.config)
+    cfg = workload_cfg(args.config, args.id_mode)
     M = cfg.M
     # R distinct global batches, resident on this GPU
     batches = [W.generate_step(W.replace(cfg, seed=cfg.seed + 1000 * rank), r, "cuda")
@@ -295,6 +344,8 @@ def run_gba(args):
     stream = torch.cuda.current_stream()
     # consecutive steps overlap (step k+1's sort during step k's row update)
     g = B.gba_for_workload(cfg, max_buf=2 * M, overlap=True)
+    if args.dense_mode == "eager":
+        g.set_eager_dense(True)  # dense gradients summed at push time
     pre = [push_args(B, cfg, b) for b in batches]
     # tokens of every step this run applies, drawn before any timing
     n_total = args.warmup + 2 * args.steps + (args.e2e_steps + 2 if args.e2e_steps > 0 else 0)
@@ -356,6 +407,10 @@ def run_gba(args):
     # roofline of the dominant kernel class: the one that must move the most
     # algorithmic bytes
     bytes_, per = alg_bytes(cfg, delta, args.steps)
+    dense_split = dense_traffic(cfg, per, args.dense_mode)
+    if args.dense_mode == "eager":  # the dense class then includes the push-time sums
+        bytes_["total"] += dense_split["bytes_per_step"] - bytes_["dense"]
+        bytes_["dense"] = dense_split["bytes_per_step"]
     classes = {"rows": kt["seg_scan"][1] + kt["row_long"][1] + kt["row_apply"][1],
                "dense": kt["dense"][1], "sort": kt["sort_hist"][1] + kt["sort_pass"][1]}
     n_launch = {"rows": kt["seg_scan"][0] + kt["row_long"][0] + kt["row_apply"][0],
@@ -433,6 +488,7 @@ def run_gba(args):
                          "timing": "CUDA events around each launch on its stream, in a second "
                                    "pass of the same steps after the timed region"},
             "kernels_ms_per_step": {n: kt[n][1] / args.steps for n in kt if n != "init"},
+            "dense_mode": dense_split,
             "per_step": per,
             "clocks": clocks,
             "gpu_launches": launches,
@@ -455,6 +511,10 @@ def main():
     ap.add_argument("--config", type=int, default=5,
                     help="workload 1-5 (default 5: the largest one that fits one GPU)")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--dense-mode", default="buffered", choices=["buffered", "eager"],
+                    help="eager: dense gradients summed into their step's accumulator at push")
+    ap.add_argument("--id-mode", default="as-configured", choices=["as-configured", "hash"],
+                    help="hash: every table an expandable hash table of 64-bit ids")
     ap.add_argument("--cpu-steps", type=int, default=3,
                     help="oracle steps timed for the cpu_baseline leg (after one warm-up step)")
     args = ap.parse_args()

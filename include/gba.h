@@ -349,6 +349,15 @@ gba_status gba_debug_keep(gba_handle* h, int32_t cap, int32_t* keep, int32_t* M)
  * this handle gives up and latches GBA_E_DEVICE_TIMEOUT (default 2e9). */
 gba_status gba_debug_set_wait_limit(gba_handle* h, int64_t ns);
 
+/* gba_debug_withhold_dense_copies - test hook for the bounded waits of K5 in
+ * the buffered dense mode: with on = 1 the dense kernel's producer issues no
+ * copies, so every consumer wait runs out after the handle's wait limit and
+ * the step reports GBA_E_DEVICE_TIMEOUT (from gba_try_apply or gba_sync); the
+ * dense parameters are then undefined and the handle is failed, as after any
+ * device timeout.  on = 0 restores normal operation.  GBA_E_ARG for other
+ * values. */
+gba_status gba_debug_withhold_dense_copies(gba_handle* h, int32_t on);
+
 /*
  * gba_selftest_wait_timeout - run the library's bounded device wait on a flag
  * that nothing sets, with the given limit, on the given stream (NULL = default
@@ -383,8 +392,7 @@ gba_status gba_selftest_wait_timeout(int64_t limit_ns, void* cuda_stream);
  * stream to finish, and returns GBA_OK, GBA_E_ID_RANGE (a DIRECT id outside
  * [0, rows)), GBA_E_DEVICE_TIMEOUT (a bounded wait of the sort gave up) or
  * GBA_E_CUDA (a CUDA call failed, or a CUDA error was already pending on the
- * calling thread; a pending error is left in place for its owner).  It must
- * not be called while the stream is being captured.  rows_out and order_out
+ * calling thread; a pending error is left in place for its owner).  rows_out and order_out
  * hold the sorted result only when GBA_OK is returned; after an error their
  * contents are undefined.
  * The first call on a device, with that device current, looks up the array's

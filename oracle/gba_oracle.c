@@ -55,7 +55,7 @@ typedef struct {
                                 ids); the tracked "rows" are then ids */
   gbao_opt opt;
   int64_t n_track;        /* number of tracked rows */
-  const int64_t* track;   /* tracked rows, strictly increasing, in [0, V) */
+  const int64_t* track;   /* tracked rows, strictly increasing (ids in id_mode 2) */
   float* w;               /* [n_track * d] */
   float* s0;              /* Adagrad accumulator or Adam first moment */
   float* s1;              /* Adam second moment (unused for Adagrad) */
@@ -242,7 +242,8 @@ static float decay_weight(const gbao_rule* rule, int64_t s, int32_t m, int32_t M
  * row_count_out[t]     (optional) per tracked row: messages containing it
  * row_kept_out[t]      (optional) per tracked row: kept occurrences
  *
- * Returns 0, or 1 when an id is out of range for a table in id_mode 0.
+ * Returns 0, or 1 when an id is out of range for a table in id_mode 0 or is
+ * the reserved id INT64_MIN in id_mode 2.
  */
 int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens,
               int32_t T, gbao_table* tables, const int64_t* const* ids,

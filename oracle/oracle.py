@@ -289,7 +289,7 @@ class OracleGBA:
                              keep_out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)), cnt_p,
                              kept_p, ctypes.byref(st))
         if rc != 0:
-            raise ValueError("id out of range for a table with id_mode 0")
+            raise ValueError("id out of range (id_mode 0) or the reserved id INT64_MIN (id_mode 2)")
         self.k += 1
         self.last_keep = keep_out[:M].copy()
         self.last_count = counts

@@ -116,6 +116,7 @@ _SIGNATURES = {
                                         ctypes.POINTER(ctypes.c_int64)]),
     "gba_debug_keep": (ctypes.c_int, [_P, ctypes.c_int32, _P, ctypes.POINTER(ctypes.c_int32)]),
     "gba_debug_set_wait_limit": (ctypes.c_int, [_P, ctypes.c_int64]),
+    "gba_debug_withhold_dense_copies": (ctypes.c_int, [_P, ctypes.c_int32]),
     "gba_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int64, _P]),
     "gba_version_string": (ctypes.c_char_p, []),
     "gba_device_binary_version": (ctypes.c_int32, []),
@@ -391,6 +392,9 @@ class GBA:
 
     def set_wait_limit(self, ns):
         check(self.L.gba_debug_set_wait_limit(self.h, int(ns)), self.h)
+
+    def withhold_dense_copies(self, on=True):
+        check(self.L.gba_debug_withhold_dense_copies(self.h, 1 if on else 0), self.h)
 
     def segments(self, cap=None):
         """Dedup output of the last step: (table, row, count, kept) numpy arrays."""

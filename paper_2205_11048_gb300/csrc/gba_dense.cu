@@ -1,6 +1,6 @@
 // K5 of the GBA aggregate-and-apply step: the dense parameters.
 //
-// g = (sum over kept messages m of grad_m) / M  (Alg. 2: weighted sum of the
+// g = (sum over kept messages m of f_m grad_m) / M  (Alg. 2: weighted sum of the
 // dense gradients divided by N_a; Appendix A: v_k = (1/M) sum g), then Adagrad
 // or Adam in place -- one pass over HBM: every kept gradient is read once, the
 // weights and optimizer state are read and written once.
@@ -61,7 +61,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
     // ---- producer
     if (lane == 0) {
       uint32_t q = 0;
-      bool ok = true;
+      bool ok = da.withhold == 0;
       for (int64_t start = r0; start < r1 && ok; start += DT) {
         const uint32_t bytes = (uint32_t)((r1 - start < DT ? r1 - start : DT) * sizeof(float));
         for (int j = 0; j < n_kept; ++j, ++q) {

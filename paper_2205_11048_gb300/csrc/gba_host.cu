@@ -155,6 +155,7 @@ struct gba_handle {
   float* d_wtab = nullptr;    // decay weights lambda^s (decay 1)
   int32_t n_wtab = 0;
   std::vector<float> h_wtab;
+  bool withhold_dense = false;  // test hook of gba_debug_withhold_dense_copies
 
   // eager dense aggregation: one compensated accumulator (hi, lo) per pending
   // global step, filled at push time
@@ -681,7 +682,11 @@ gba_status push_common(gba_handle* h, int64_t token, const gba_sparse_grad* per_
         src = h->d_stage_dense;
       }
       float* hi = h->d_acc + (size_t)gr.slot * 2 * h->D_pad;
-      launch_dense_accumulate(hi, hi + h->D_pad, src, h->D, f, !gr.has_sum, h->num_sms, h->stream);
+      {
+        Timed tm(h, GBA_K_DENSE, h->stream);
+        launch_dense_accumulate(hi, hi + h->D_pad, src, h->D, f, !gr.has_sum, h->num_sms,
+                                h->stream);
+      }
       GBA_CUDA(h, cudaGetLastError());
       gr.has_sum = true;
     }
@@ -1046,7 +1051,8 @@ int32_t gba_try_apply(gba_handle* h) {
     if (h->D <= 0) return;
     const double p1 = h->dbpow1 * (double)h->dense_opt.beta1;
     const double p2 = h->dbpow2 * (double)h->dense_opt.beta2;
-    DenseArgs da{h->dw, h->ds0, h->ds1, h->D, M, make_opt_step(h->dense_opt, p1, p2)};
+    DenseArgs da{h->dw, h->ds0, h->ds1, h->D, M, make_opt_step(h->dense_opt, p1, p2),
+                 h->withhold_dense ? 1 : 0};
     cudaEventRecord(h->ev_hist[b], h->sorts);
     cudaStreamWaitEvent(h->side, h->ev_hist[b], 0);
     if (h->eager) {  // the step's sum was accumulated at push time
@@ -1410,6 +1416,12 @@ gba_status gba_debug_keep(gba_handle* h, int32_t cap, int32_t* keep, int32_t* M)
 gba_status gba_debug_set_wait_limit(gba_handle* h, int64_t ns) {
   if (!h || ns < 0) return GBA_E_ARG;
   h->wait_ns = ns;
+  return GBA_OK;
+}
+
+gba_status gba_debug_withhold_dense_copies(gba_handle* h, int32_t on) {
+  if (!h || (on != 0 && on != 1)) return GBA_E_ARG;
+  h->withhold_dense = on != 0;
   return GBA_OK;
 }
 

@@ -417,6 +417,8 @@ struct DenseArgs {
   int64_t D;
   int32_t M;
   OptStep opt;
+  int32_t withhold = 0;  // test hook: the producer issues no copies, so every
+                         // consumer wait runs out and reports ERR_TIMEOUT
 };
 
 size_t dense_smem_bytes();

@@ -12,8 +12,7 @@
 //    bytes; every GPU that loads the library keeps it until the process exits.
 //  - The first call on a device (with that device current) looks up the
 //    array's device address with cudaGetSymbolAddress.
-//  - The call is synchronous: it waits for its stream before returning, so it
-//    cannot be captured into a CUDA graph.
+//  - The call is synchronous: it waits for its stream before returning.
 //  - All calls share the one array and it keeps the previous call's contents.
 //    The per-call counters are cleared at the start of each call; calls whose
 //    work overlaps on the GPU (two streams, or two host threads) race.

@@ -16,19 +16,20 @@
 //               writes the address of its gradient row (and its weight) into
 //               a list sorted by row.  Rows that cross tiles need no special
 //               care: a row's counts are differences of prefixes.
-//  k_row_apply  One lane group per row (L lanes, 16-byte pieces when the width
-//               is a multiple of 4), grid-stride over the rows: the row's kept
-//               gradients are summed in sorted order with compensated (TwoSum)
-//               arithmetic, divided by the denominator and applied with the
-//               row's weights and state, which are loaded together with the
-//               gradients; the next row's list entries are loaded one row
-//               ahead.  Rows with more than LONG_ROW kept occurrences are
-//               handed to the next kernel.
-//  k_row_long   Those rows in chunks of LONG_CHUNK kept occurrences, one block
-//               per chunk: every lane group sums a contiguous part, the parts
-//               are merged in order, and a row split into several chunks is
-//               finished by the block that completes its last chunk, merging
-//               the chunk sums in chunk order.
+//  k_row_apply_staged  Rows with at most LONG_ROW kept occurrences (widths a
+//               multiple of 4): one lane group per row, grid-stride over the
+//               rows; the row's records, kept-list entries, weights, state and
+//               gradient rows are copied into shared memory by a three-level
+//               cp.async pipeline several rows ahead, then the kept gradients
+//               are summed in sorted order with compensated (TwoSum)
+//               arithmetic, divided by the denominator and applied.
+//  k_row_apply  The same with register-held rows, for other widths.
+//  k_row_long   Rows with more kept occurrences, in chunks of LONG_CHUNK of
+//               them, one warp per chunk claimed in list order: the warp's
+//               lane groups sum contiguous parts that are merged in order,
+//               and a row split into several chunks is finished by the warp
+//               that completes its last chunk, merging the chunk sums in
+//               chunk order.
 //
 // Every summation order is fixed (sorted order, then fixed parts and chunks),
 // so results are bit-identical run to run; no float atomics anywhere.

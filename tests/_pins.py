@@ -353,23 +353,27 @@ def pin_order_invariance(L, seed=11):
 
 
 # ---------------------------------------------------------------------------
-def brute_force_run(specs, D, dense_opt, G, iota, steps, seed):
+def brute_force_run(specs, D, dense_opt, G, iota, steps, seed, keys=None):
     """A literal restatement for tiny inputs: enumerate every (message,
     occurrence) pair, keep a dictionary per row, and round to float32 after
-    every operation in the stated order."""
+    every operation in the stated order.  keys[t] lists table t's row keys
+    (default: 0..rows-1); a key x starts from the initial values of element
+    x*d + j (modulo 2^64), so keys may be arbitrary 64-bit ids."""
     f32 = np.float32
-    st = {}
     t_specs = specs
+    if keys is None:
+        keys = [range(sp.rows) for sp in t_specs]
     init_w = {}
     for t, sp in enumerate(t_specs):
-        for x in range(sp.rows):
+        for x in keys[t]:
             for j in range(sp.dim):
-                init_w[(t, x, j)] = f32(O.init_weight(seed, O.table_tag(t), x * sp.dim + j))
+                e = (int(x) * sp.dim + j) % 2**64
+                init_w[(t, int(x), j)] = f32(O.init_weight(seed, O.table_tag(t), e))
     W = dict(init_w)
     S0 = {key: (f32(t_specs[key[0]].opt.init_acc) if t_specs[key[0]].opt.kind == O.ADAGRAD
                 else f32(0)) for key in W}
     S1 = {key: f32(0) for key in W}
-    ver = {(t, x): 0 for t, sp in enumerate(t_specs) for x in range(sp.rows)}
+    ver = {(t, int(x)): 0 for t in range(len(t_specs)) for x in keys[t]}
     DW = [f32(O.init_weight(seed, O.dense_tag(), e)) for e in range(D)]
     DS0 = [f32(dense_opt.init_acc) if dense_opt.kind == O.ADAGRAD else f32(0)] * D
     DS1 = [f32(0)] * D
@@ -465,9 +469,81 @@ def pin_brute_force(L, seed=21):
         assert orc.dense.s0.tolist() == [float(v) for v in DS0]
 
 
+def pin_hash_ids(L, seed=41):
+    """Tables of arbitrary 64-bit ids (id mode 2): with ids in [0, V) they
+    evolve bit for bit as DIRECT tables; with ids anywhere in the int64 range
+    (negative, beyond 2^32, repeated within a message) they agree bit for bit
+    with the brute-force restatement keyed by id; the reserved id INT64_MIN
+    is an error."""
+    rng = np.random.default_rng(seed)
+    V, d, D, M = 6, 3, 2, 4
+    for kind in (O.ADAGRAD, O.ADAM):
+        # small ids: the same as row = id
+        direct = O.OracleGBA([O.TableSpec(V, d, O.OptSpec(kind, 0.03))], D,
+                             O.OptSpec(kind, 0.01), M, iota=1, seed=5, library=L)
+        hashed = O.OracleGBA([O.TableSpec(V, d, O.OptSpec(kind, 0.03), id_mode=2)], D,
+                             O.OptSpec(kind, 0.01), M, iota=1, seed=5, library=L,
+                             track_rows=[np.arange(V, dtype=np.int64)])
+        for s in range(3):
+            for m in range(M):
+                n = int(rng.integers(0, 5))
+                msg = O.Message(max(0, s - int(rng.integers(0, 3))), 1,
+                                [rng.integers(0, V, n).astype(np.int64)],
+                                [(rng.standard_normal((n, d)) * .5).astype(np.float32)],
+                                (rng.standard_normal(D) * .5).astype(np.float32))
+                direct.push(msg)
+                hashed.push(msg)
+            assert direct.try_apply() == 1 and hashed.try_apply() == 1
+        assert direct.tables[0].w.tobytes() == hashed.tables[0].w.tobytes()
+        assert direct.tables[0].s0.tobytes() == hashed.tables[0].s0.tobytes()
+        assert direct.tables[0].ver.tolist() == hashed.tables[0].ver.tolist()
+
+        # arbitrary ids against the brute force keyed by id
+        pool = np.array([-2**63 + 1, -7, 0, 3, 2**33 + 5, 2**62 + 11], np.int64)
+        spec = O.TableSpec(len(pool), d, O.OptSpec(kind, 0.03), id_mode=2)
+        dopt = O.OptSpec(kind, 0.01)
+        orc = O.OracleGBA([spec], D, dopt, M, iota=1, seed=9, library=L,
+                          track_rows=[np.sort(pool)])
+        steps = []
+        for s in range(3):
+            batch = []
+            for m in range(M):
+                n = int(rng.integers(0, 5))
+                ids = pool[rng.integers(0, len(pool), n)]
+                batch.append(O.Message(max(0, s - int(rng.integers(0, 3))), 1, [ids],
+                                       [(rng.standard_normal((n, d)) * .5).astype(np.float32)],
+                                       (rng.standard_normal(D) * .5).astype(np.float32)))
+            steps.append(batch)
+            for msg in batch:
+                orc.push(msg)
+            assert orc.try_apply() == 1
+        W, S0, S1, ver, DW, _, _ = brute_force_run([spec], D, dopt, M, 1, steps, 9,
+                                                    keys=[sorted(int(x) for x in pool)])
+        w = orc.tables[0].w.reshape(-1, d)
+        s0 = orc.tables[0].s0.reshape(-1, d)
+        for r, x in enumerate(sorted(int(x) for x in pool)):
+            assert orc.tables[0].ver[r] == ver[(0, x)], ("ver", kind, x)
+            for j in range(d):
+                assert w[r, j] == W[(0, x, j)], ("w", kind, x, j)
+                assert s0[r, j] == S0[(0, x, j)], ("s0", kind, x, j)
+        assert orc.dense.w.tolist() == [float(v) for v in DW]
+
+    # the reserved id
+    orc = O.OracleGBA([O.TableSpec(4, 1, id_mode=2)], 1, O.OptSpec(), 1, library=L,
+                      track_rows=[np.arange(4, dtype=np.int64)])
+    orc.push(O.Message(0, 1, [np.array([-2**63], np.int64)], [np.ones((1, 1), np.float32)],
+                       np.ones(1, np.float32)))
+    try:
+        orc.try_apply()
+    except ValueError:
+        pass
+    else:
+        raise AssertionError("the reserved id was accepted")
+
+
 ALL_PINS = [pin_hand_adagrad, pin_hand_rule_options, pin_hand_decay_variants,
             pin_decay_special_cases, pin_hand_adam, pin_sync_closed_form, pin_decay_boundary,
-            pin_fifo_prefix, pin_order_invariance, pin_brute_force]
+            pin_fifo_prefix, pin_order_invariance, pin_brute_force, pin_hash_ids]
 
 
 def pin_init_published(L):

@@ -442,6 +442,44 @@ def test_tiny_wait_limit_in_dense_is_reported_or_harmless():
     g2.close()
 
 
+def test_dense_waits_run_out_when_copies_are_withheld():
+    """K5's bounded waits, forced: the producer issues no copies, so every
+    consumer waits on a stage nothing fills; after the 1 ms limit each wait
+    gives up, the step reports GBA_E_DEVICE_TIMEOUT, the handle stays failed,
+    and the context is still usable (a fresh handle applies a step that
+    matches the oracle's dense update)."""
+    D, M = 1_000_003, 4
+    dense_opt = B.opt_desc(W.ADAGRAD, 0.01)
+    gen = torch.Generator(device="cuda").manual_seed(13)
+    grads = [torch.randn(D, generator=gen, device="cuda") * 0.01 for _ in range(M)]
+    g = B.GBA([], D, dense_opt, M, 2 * M, seed=3)
+    g.set_wait_limit(1_000_000)
+    g.withhold_dense_copies(True)
+    for i in range(M):
+        g.push_ref(0, [], [], grads[i], 1)
+    rc = g.L.gba_try_apply(g.h)
+    if rc == 1:
+        rc = g.L.gba_sync(g.h)
+    assert rc == B.GBA_E_DEVICE_TIMEOUT
+    assert g.L.gba_try_apply(g.h) != 1  # the handle stays failed
+    g.close()
+    torch.cuda.synchronize()
+    g2 = B.GBA([], D, dense_opt, M, 2 * M, seed=3)
+    for i in range(M):
+        g2.push_ref(0, [], [], grads[i], 1)
+    assert g2.try_apply() == 1
+    g2.sync()
+    w, _, _ = g2.dense()
+    orc = O.OracleGBA([], D, O.OptSpec(O.ADAGRAD, 0.01), M, seed=3,
+                      track_dense=np.arange(0, D, 997, dtype=np.int64))
+    for i in range(M):
+        orc.push(O.Message(0, 1, [], [], grads[i].cpu().numpy()))
+    assert orc.try_apply() == 1
+    got = w.cpu().numpy()[np.arange(0, D, 997)]
+    np.testing.assert_allclose(got, orc.dense.w, rtol=1e-5, atol=1e-7)
+    g2.close()
+
+
 def test_device_code_is_sm103a():
     """The kernels run from sm_103a device code on this GPU."""
     assert B.load().gba_device_binary_version() == 103

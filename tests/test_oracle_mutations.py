@@ -59,6 +59,10 @@ MUTATIONS = [
      "if (m < rule->drop_latest) return 0.0f;", 0),
     ("hopbw-off-by-one", "if (m >= M - rule->drop_latest) return 0.0f;",
      "if (m > M - rule->drop_latest) return 0.0f;", 0),
+    ("hash-reserved-id-accepted", "if (id == INT64_MIN) { err = 1; continue; }",
+     "if (id == INT64_MIN) { x = id; }", 0),
+    ("hash-ids-folded", "  /* the reserved id */\n          x = id;",
+     "  /* the reserved id */\n          x = (int64_t)((uint64_t)id % (uint64_t)tb->V);", 0),
 ]
 
 
