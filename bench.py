@@ -46,12 +46,19 @@ def peaks():
     return 6800.0, "fallback"
 
 
-def workload_cfg(n, id_mode="as-configured"):
+def workload_cfg(n, id_mode="as-configured", rows=None, dense=None):
     """Workload n; id_mode "hash" turns every table into an expandable hash
     table of 64-bit ids (initial capacity: the next power of two at or above
-    twice its rows)."""
+    twice its rows).  rows / dense shrink the tables' rows and the dense size
+    while keeping the message, id and staleness structure: a case of the same
+    shape small enough for a multi-pass profiler capture."""
     from paper_2205_11048_gb300 import workload as W
     cfg = W.config(n)
+    if rows is not None or dense is not None:
+        r = rows if rows is not None else cfg.tables[0].rows
+        D = dense if dense is not None else cfg.D
+        cfg = W.replace(cfg, name=f"{cfg.name}-shaped-{r}x{cfg.tables[0].dim}-D{D}", D=D,
+                        tables=tuple(W.replace(t, rows=r) for t in cfg.tables))
     if id_mode == "hash":
         def cap(r):
             c = 1024
@@ -61,6 +68,10 @@ def workload_cfg(n, id_mode="as-configured"):
         cfg = W.replace(cfg, name=cfg.name + "-hash-ids",
                         tables=tuple(W.replace(t, id_mode=W.HASH, rows=cap(t.rows))
                                      for t in cfg.tables))
+        state = sum(t.rows * (4 * t.dim * (2 if t.opt.kind == 0 else 3) + 12) for t in cfg.tables)
+        if state > 150e9:
+            raise SystemExit(f"--id-mode hash: {state / 1e9:.0f} GB of table state at the initial "
+                             "capacity; use --shape-rows for a smaller case")
     return cfg
 
 
@@ -288,7 +299,7 @@ def run_reference(args):
     if rank != 0:
         return
     from paper_2205_11048_gb300 import workload as W
-    cfg = workload_cfg(args.config, args.id_mode)
+    cfg = workload_cfg(args.config, args.id_mode, args.shape_rows, args.shape_dense)
     batches = [W.generate_step(cfg, r, "cpu") for r in range(R_BATCHES)]
     sps, sample = oracle_rate(cfg, batches, args.warmup, args.steps)
     line = {"impl": "reference", "metric": METRIC, "value": sps, "unit": "steps/s",
@@ -335,7 +346,7 @@ def run_gba(args):
         __graft_entry__.build()
     L = B.load()
 
-    cfg = workload_cfg(args.config, args.id_mode)
+    cfg = workload_cfg(args.config, args.id_mode, args.shape_rows, args.shape_dense)
     M = cfg.M
     # R distinct global batches, resident on this GPU
     batches = [W.generate_step(W.replace(cfg, seed=cfg.seed + 1000 * rank), r, "cuda")
@@ -505,7 +516,7 @@ def run_gba(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=300)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="gba", choices=["gba", "reference"])
     ap.add_argument("--config", type=int, default=5,
@@ -515,6 +526,10 @@ def main():
                     help="eager: dense gradients summed into their step's accumulator at push")
     ap.add_argument("--id-mode", default="as-configured", choices=["as-configured", "hash"],
                     help="hash: every table an expandable hash table of 64-bit ids")
+    ap.add_argument("--shape-rows", type=int, default=None,
+                    help="rows of every table (profiling case of the same shape)")
+    ap.add_argument("--shape-dense", type=int, default=None,
+                    help="dense parameters (profiling case of the same shape)")
     ap.add_argument("--cpu-steps", type=int, default=3,
                     help="oracle steps timed for the cpu_baseline leg (after one warm-up step)")
     args = ap.parse_args()

@@ -6,13 +6,11 @@
 // weights and optimizer state are read and written once.
 //
 // Each persistent CTA walks an equal contiguous share of the parameters in
-// tiles of up to 2048.  A producer warp streams
-// the tile's slice of every kept message into a ring of shared-memory stages
-// with 1-D bulk async copies (cp.async.bulk, completion counted on an mbarrier
-// per stage); eight consumer warps sum the slices with compensated (TwoSum)
-// float arithmetic, release each stage on an "empty" mbarrier, and finish the
-// tile
-// with the optimizer.  Every mbarrier wait is bounded in time; a wait that
+// tiles of up to DT.  A producer warp streams the tile's slice of every kept
+// message into a ring of shared-memory stages with 1-D bulk async copies
+// (cp.async.bulk, completion counted on an mbarrier per stage); eight consumer
+// warps sum the slices with compensated (TwoSum) float arithmetic, release each
+// stage on an "empty" mbarrier, and finish the tile with the optimizer.  Every mbarrier wait is bounded in time; a wait that
 // gives up latches ERR_TIMEOUT, the CTA stops issuing copies, waits (bounded)
 // for the copies it already issued, and exits.
 #include "gba_internal.cuh"
@@ -21,10 +19,18 @@ namespace gba {
 
 namespace {
 
-constexpr int DT = 2048;           // parameters per tile
-constexpr int STAGES = 8;          // 8 KB each
-constexpr int CONSUMER_WARPS = 8;  // 256 threads, two float4 each
-constexpr int HALF = DT / 2;       // thread c owns [4c, 4c+4) and [HALF+4c, HALF+4c+4)
+#ifndef GBA_DENSE_TILE
+#define GBA_DENSE_TILE 2048
+#endif
+#ifndef GBA_DENSE_STAGES
+#define GBA_DENSE_STAGES 8
+#endif
+constexpr int DT = GBA_DENSE_TILE;       // parameters per tile
+constexpr int STAGES = GBA_DENSE_STAGES;  // DT floats each
+constexpr int CONSUMER_WARPS = 8;        // 256 threads
+constexpr int HALF = CONSUMER_WARPS * 32 * 4;  // floats of one float4 per consumer thread
+constexpr int PER = DT / HALF;  // thread c owns [h*HALF + 4c, h*HALF + 4c + 4), h < PER
+static_assert(DT % HALF == 0, "a tile is a whole number of float4 rows of the consumers");
 constexpr int DENSE_THREADS = (CONSUMER_WARPS + 1) * 32;
 
 __global__ void __launch_bounds__(DENSE_THREADS)
@@ -88,18 +94,18 @@ __global__ void __launch_bounds__(DENSE_THREADS)
       }
     }
   } else {
-    // ---- consumers: thread c owns parameters [4c, 4c + 4) and
-    // [HALF + 4c, HALF + 4c + 4) of each tile
+    // ---- consumers: thread c owns parameters [h*HALF + 4c, h*HALF + 4c + 4)
+    // of each tile, h < PER
     const int c = tid;
     const float Mf = (float)da.M;
     uint32_t q = 0;
     for (int64_t start = r0; start < r1; start += DT) {
       const int64_t n = r1 - start < DT ? r1 - start : DT;
-      bool mine[2];
-      int64_t e[2];
-      float4 w[2], s0[2], s1[2];
+      bool mine[PER];
+      int64_t e[PER];
+      float4 w[PER], s0[PER], s1[PER];
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
+      for (int h = 0; h < PER; ++h) {
         const int64_t off = (int64_t)h * HALF + (int64_t)c * 4;
         mine[h] = off < n;
         e[h] = start + off;
@@ -110,9 +116,9 @@ __global__ void __launch_bounds__(DENSE_THREADS)
           if (da.opt.kind == 1) s1[h] = *reinterpret_cast<const float4*>(da.s1 + e[h]);
         }
       }
-      CSum acc[8];
+      CSum acc[4 * PER];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) acc[i] = CSum{0.f, 0.f};
+      for (int i = 0; i < 4 * PER; ++i) acc[i] = CSum{0.f, 0.f};
       bool aborted = false;
       for (int j = 0; j < n_kept; ++j, ++q) {
         const int stage = (int)(q % STAGES);
@@ -130,7 +136,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
         }
         if (a.decay == 0) {
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
+          for (int h = 0; h < PER; ++h) {
             if (mine[h]) {
               const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT +
                                                                 h * HALF + 4 * c);
@@ -143,7 +149,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
         } else {  // weighted: f_m * g with the product's rounding error kept
           const float f = sc.fw[j];
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
+          for (int h = 0; h < PER; ++h) {
             if (mine[h]) {
               const float4 v = *reinterpret_cast<const float4*>(stage_buf + (size_t)stage * DT +
                                                                 h * HALF + 4 * c);
@@ -159,7 +165,7 @@ __global__ void __launch_bounds__(DENSE_THREADS)
       }
       if (aborted || __shfl_sync(0xffffffffu, *(volatile int*)&s_abort, 0) != 0) break;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
+      for (int h = 0; h < PER; ++h) {
         if (!mine[h]) continue;
         float wv[4] = {w[h].x, w[h].y, w[h].z, w[h].w},
               a0[4] = {s0[h].x, s0[h].y, s0[h].z, s0[h].w},
@@ -261,7 +267,15 @@ void launch_dense(const StepArgs& a, const DenseArgs& da, StepScratch sc, ErrSin
                   int64_t wait_ns, int num_sms, cudaStream_t s) {
   const size_t smem = dense_smem_bytes();
   const int64_t n_tiles = ((da.D & ~3ll) + DT - 1) / DT;
-  int64_t grid = (int64_t)num_sms * 3;
+  static const int bps = [&]() {  // persistent: as many CTAs as fit on an SM
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, k_dense_apply, DENSE_THREADS, smem) !=
+            cudaSuccess ||
+        b < 1)
+      b = 1;
+    return b;
+  }();
+  int64_t grid = (int64_t)num_sms * bps;
   if (grid > n_tiles) grid = n_tiles;
   if (grid < 1) grid = 1;
   k_dense_apply<<<(unsigned)grid, DENSE_THREADS, smem, s>>>(a, da, sc, err, wait_ns);

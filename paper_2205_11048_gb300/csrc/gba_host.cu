@@ -82,6 +82,10 @@ size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 }  // namespace
 
+#ifndef GBA_LONG_STREAM
+#define GBA_LONG_STREAM 0
+#endif
+
 struct gba_handle {
   int device = 0;
   int num_sms = 152;
@@ -90,6 +94,8 @@ struct gba_handle {
   cudaStream_t side = nullptr;   // dense update
   cudaStream_t sorts = nullptr;   // message weights, histogram, sort passes
   cudaStream_t applys = nullptr;  // segment-sum and row update
+  cudaStream_t longs = nullptr;   // long rows (when run beside the short rows)
+  cudaEvent_t ev_classified = nullptr, ev_longs = nullptr;
   bool overlap = false;           // consecutive steps may run concurrently
   cudaEvent_t ev_pushes = nullptr;
   cudaEvent_t ev_hist[SLOTS] = {}, ev_sorted[SLOTS] = {}, ev_applied[SLOTS] = {},
@@ -145,6 +151,7 @@ struct gba_handle {
   float* d_kw = nullptr;                   // kept weights
   unsigned long long* d_scan_status = nullptr;
   uint4* d_long_rows = nullptr;
+  uint4* d_small_rows = nullptr;
   uint32_t* d_long_done = nullptr;
   uint2* d_items = nullptr;
   float* d_part_hi = nullptr;
@@ -288,6 +295,7 @@ void free_all(gba_handle* h) {
   cudaSetDevice(h->device);
   if (h->sorts) cudaStreamSynchronize(h->sorts);
   if (h->applys) cudaStreamSynchronize(h->applys);
+  if (h->longs) cudaStreamSynchronize(h->longs);
   if (h->side) cudaStreamSynchronize(h->side);
   if (h->stream) cudaStreamSynchronize(h->stream);
   for (auto& t : h->tables) {
@@ -323,7 +331,8 @@ void free_all(gba_handle* h) {
   }
   for (void* p : {(void*)h->d_rr, (void*)h->d_kl, (void*)h->d_kw, (void*)h->d_scan_status,
                   (void*)h->d_long_rows, (void*)h->d_long_done, (void*)h->d_items,
-                  (void*)h->d_part_hi, (void*)h->d_part_lo, (void*)h->d_seg_total})
+                  (void*)h->d_part_hi, (void*)h->d_part_lo, (void*)h->d_seg_total,
+                  (void*)h->d_small_rows})
     cudaFree(p);
   cudaFree(h->d_err);
   cudaFree(h->d_wtab);
@@ -339,6 +348,9 @@ void free_all(gba_handle* h) {
   }
   for (auto e : h->event_pool) cudaEventDestroy(e);
   if (h->ev_pushes) cudaEventDestroy(h->ev_pushes);
+  if (h->ev_classified) cudaEventDestroy(h->ev_classified);
+  if (h->ev_longs) cudaEventDestroy(h->ev_longs);
+  if (h->longs) cudaStreamDestroy(h->longs);
   if (h->side) cudaStreamDestroy(h->side);
   if (h->sorts) cudaStreamDestroy(h->sorts);
   if (h->applys) cudaStreamDestroy(h->applys);
@@ -346,8 +358,9 @@ void free_all(gba_handle* h) {
 }
 
 cudaError_t sync_all(gba_handle* h) {
-  cudaError_t e[4] = {cudaStreamSynchronize(h->sorts), cudaStreamSynchronize(h->applys),
-                      cudaStreamSynchronize(h->side), cudaStreamSynchronize(h->stream)};
+  cudaError_t e[5] = {cudaStreamSynchronize(h->sorts), cudaStreamSynchronize(h->applys),
+                      cudaStreamSynchronize(h->longs), cudaStreamSynchronize(h->side),
+                      cudaStreamSynchronize(h->stream)};
   for (cudaError_t x : e)
     if (x != cudaSuccess) return x;
   return cudaSuccess;
@@ -516,13 +529,14 @@ gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
     // long rows and their chunks
     for (void* p : {(void*)h->d_rr, (void*)h->d_kl, (void*)h->d_kw, (void*)h->d_scan_status,
                     (void*)h->d_long_rows, (void*)h->d_long_done, (void*)h->d_items,
-                    (void*)h->d_part_hi, (void*)h->d_part_lo})
+                    (void*)h->d_part_hi, (void*)h->d_part_lo, (void*)h->d_small_rows})
       cudaFree(p);
     h->d_rr = nullptr;
     h->d_kl = nullptr;
     h->d_kw = h->d_part_hi = h->d_part_lo = nullptr;
     h->d_scan_status = nullptr;
     h->d_long_rows = nullptr;
+    h->d_small_rows = nullptr;
     h->d_long_done = nullptr;
     h->d_items = nullptr;
     const int64_t stiles = scan_tiles(cap);
@@ -535,6 +549,7 @@ gba_status ensure_step_capacity(gba_handle* h, int64_t N) {
     GBA_CUDA(h, cudaMalloc(&h->d_scan_status, (size_t)stiles * 4 * sizeof(unsigned long long)));
     GBA_CUDA(h, cudaMemset(h->d_scan_status, 0, (size_t)stiles * 4 * sizeof(unsigned long long)));
     GBA_CUDA(h, cudaMalloc(&h->d_long_rows, (size_t)long_cap * sizeof(uint4)));
+    GBA_CUDA(h, cudaMalloc(&h->d_small_rows, (size_t)long_cap * sizeof(uint4)));
     GBA_CUDA(h, cudaMalloc(&h->d_long_done, (size_t)long_cap * sizeof(uint32_t)));
     GBA_CUDA(h, cudaMalloc(&h->d_items, (size_t)items_cap * sizeof(uint2)));
     GBA_CUDA(h, cudaMalloc(&h->d_part_hi, (size_t)parts_cap * h->d_max * sizeof(float)));
@@ -774,7 +789,10 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
   if (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&h->sorts, cudaStreamNonBlocking) != cudaSuccess ||
       cudaStreamCreateWithFlags(&h->applys, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_pushes, cudaEventDisableTiming) != cudaSuccess)
+      cudaStreamCreateWithFlags(&h->longs, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_pushes, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_classified, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_longs, cudaEventDisableTiming) != cudaSuccess)
     return fail(GBA_E_CUDA);
   for (int b = 0; b < SLOTS; ++b)
     for (cudaEvent_t* e : {&h->ev_hist[b], &h->ev_sorted[b], &h->ev_applied[b], &h->ev_densed[b]})
@@ -1133,11 +1151,33 @@ int32_t gba_try_apply(gba_handle* h) {
       so.part_hi = h->d_part_hi;
       so.part_lo = h->d_part_lo;
       so.pstride = h->d_max;
+      so.small_rows = h->d_small_rows;
+      so.n_small = sc.seg_ticket + 8 * t + 5;
+      so.small_ticket = sc.seg_ticket + 8 * t + 6;
       {
         Timed tm(h, GBA_K_SEG_SCAN, h->applys);
         launch_seg_scan(a, tb, so, h->d_keys[b][final_buf], h->d_vals[b][final_buf], h->d_stats,
                         sink, h->wait_ns, h->applys);
       }
+      {
+        Timed tm(h, GBA_K_SEG_SCAN, h->applys);
+        launch_row_classify(a, tb, so, sink, h->num_sms, h->applys);
+      }
+#if GBA_LONG_STREAM
+      // long rows on their own stream, next to the short rows
+      cudaEventRecord(h->ev_classified, h->applys);
+      cudaStreamWaitEvent(h->longs, h->ev_classified, 0);
+      {
+        Timed tm(h, GBA_K_ROW_LONG, h->longs);
+        launch_row_long(a, tb, so, h->d_stats, sink, h->num_sms, h->longs);
+      }
+      {
+        Timed tm(h, GBA_K_ROW_APPLY, h->applys);
+        launch_row_apply(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
+      }
+      cudaEventRecord(h->ev_longs, h->longs);
+      cudaStreamWaitEvent(h->applys, h->ev_longs, 0);
+#else
       {
         Timed tm(h, GBA_K_ROW_APPLY, h->applys);
         launch_row_apply(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
@@ -1146,6 +1186,7 @@ int32_t gba_try_apply(gba_handle* h) {
         Timed tm(h, GBA_K_ROW_LONG, h->applys);
         launch_row_long(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
       }
+#endif
     }
   }
   if (N == 0) {

@@ -305,6 +305,16 @@ __device__ __forceinline__ void csum_add_prod(CSum& c, float f, float g) {
   c.lo = __fadd_rn(c.lo, __fadd_rn(t, e));
 }
 
+// A kept term of a weighted sum.  With decay strategy 0 every kept weight is
+// exactly 1 and the term is added by csum_add, which gives what csum_add_prod
+// gives for f = 1 (the product and its error are g and 0) with fewer operations.
+__device__ __forceinline__ void csum_add_w(CSum& c, bool unit, float f, float g) {
+  if (unit)
+    csum_add(c, g);
+  else
+    csum_add_prod(c, f, g);
+}
+
 // Accumulated statistics (device).
 struct DevStats {
   unsigned long long steps, msgs_kept, msgs_dropped, dense_stale_sum, dense_stale_max, pairs,
@@ -386,6 +396,9 @@ struct SegOut {
   float* part_hi;              // [n_parts][pstride] compensated chunk sums
   float* part_lo;
   int32_t pstride;
+  uint4* small_rows;           // [n_small] (row, first kept, kept count, denominator bits)
+  uint32_t* n_small;           // long rows of at most SMALL_MAX kept occurrences (cleared by K1)
+  uint32_t* small_ticket;      // small rows claimed by the long-row kernel (cleared by K1)
 };
 
 // Rows with at most LONG_ROW kept occurrences are applied by one lane group
@@ -396,7 +409,16 @@ constexpr int LONG_ROW = 4;
 #define GBA_LONG_CHUNK 128
 #endif
 constexpr int LONG_CHUNK = GBA_LONG_CHUNK;
-constexpr int SCAN_TILE = 2048;
+// Long rows of at most SMALL_MAX kept occurrences are applied by one lane
+// group each, with all their gradient rows staged in shared memory.
+#ifndef GBA_SMALL_MAX
+#define GBA_SMALL_MAX 32
+#endif
+constexpr int SMALL_MAX = GBA_SMALL_MAX;
+#ifndef GBA_SCAN_TILE
+#define GBA_SCAN_TILE 2048
+#endif
+constexpr int SCAN_TILE = GBA_SCAN_TILE;  // sorted positions per segment-scan tile
 
 int64_t scan_tiles(int64_t N);
 
@@ -409,6 +431,10 @@ void launch_row_apply(const StepArgs& a, const SegTable& tb, const SegOut& so, D
 
 void launch_row_long(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
                      ErrSink err, int num_sms, cudaStream_t s);
+
+// Lists the long rows and their chunks (after the scan, before both row kernels).
+void launch_row_classify(const StepArgs& a, const SegTable& tb, const SegOut& so, ErrSink err,
+                         int num_sms, cudaStream_t s);
 
 struct DenseArgs {
   float* w;

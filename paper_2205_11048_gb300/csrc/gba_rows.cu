@@ -85,6 +85,24 @@ __device__ __forceinline__ int message_of_any(const uint32_t* off, int M, uint32
   return lo;
 }
 
+// The same, starting from the message an even split would give (exact when
+// every message holds the same number of ids, as with one-hot fields; scale
+// is M over the table's occurrences) and falling back to the binary search
+// when that guess is more than two messages off.
+__device__ __forceinline__ int message_of(const uint32_t* off, int M, uint32_t x, float scale) {
+  int m = (int)((float)x * scale);
+  m = m < 0 ? 0 : (m < M - 1 ? m : M - 1);
+#pragma unroll
+  for (int s = 0; s < 2; ++s) {
+    if (m > 0 && off[m] > x)
+      --m;
+    else if (m + 1 < M && off[m + 1] <= x)
+      ++m;
+  }
+  if (off[m] <= x && (m + 1 >= M || off[m + 1] > x)) return m;
+  return message_of_any(off, M, x);
+}
+
 // Denominator of a row's weighted sum (Alg. 2: messages that encountered the
 // row; or the messages whose occurrence was kept; or all M messages).
 __device__ __forceinline__ float row_denominator(int mode, uint32_t c_all, uint32_t c_kept, int M) {
@@ -95,6 +113,9 @@ __device__ __forceinline__ float row_denominator(int mode, uint32_t c_all, uint3
 // ---------------------------------------------------------------------------
 // k_seg_scan
 // ---------------------------------------------------------------------------
+#ifndef GBA_LOOKBACK_SLEEP_NS
+#define GBA_LOOKBACK_SLEEP_NS 64
+#endif
 #ifndef GBA_SCAN_MINB
 #define GBA_SCAN_MINB 2
 #endif
@@ -150,6 +171,7 @@ __global__ void __launch_bounds__(SCAN_THREADS, GBA_SCAN_MINB)
   const uint32_t n_t = (uint32_t)Nt;
   const uint32_t v_t = (uint32_t)tb.rows;
   const int hop_limit = M - a.drop_latest;  // messages at or past this index are dropped
+  const float mscale = (float)M / (float)(n_t > 0u ? n_t : 1u);
 
   // ---- pass 1: decide every position of this thread's 8 (blocked layout)
   const int i0 = tid * SCAN_ITEMS;
@@ -163,7 +185,7 @@ __global__ void __launch_bounds__(SCAN_THREADS, GBA_SCAN_MINB)
   int m_prev = -1;
   if (i0 < n_valid && s_k[SCAN_PAD(i0)] != NO_KEY) {  // message of the position before
     const uint32_t o_t = (uint32_t)((int64_t)s_v[SCAN_PAD(i0)] - nbase);
-    if (o_t < n_t) m_prev = message_of_any(off, M, o_t);
+    if (o_t < n_t) m_prev = message_of(off, M, o_t, mscale);
   }
   // the rows' step tags first, all eight loads in flight together (positions
   // of one row read the same tag, so only a row's first read reaches DRAM)
@@ -189,7 +211,7 @@ __global__ void __launch_bounds__(SCAN_THREADS, GBA_SCAN_MINB)
         raise_error(err, ERR_INTERNAL);  // cannot happen for a correctly sorted array
         continue;
       }
-      const int m = message_of_any(off, M, o_t);
+      const int m = message_of(off, M, o_t, mscale);
       const int64_t tok = cached ? s_tok[m] : a.tokens[m];
       const int64_t ref = a.row_staleness == 0 ? (int64_t)tg_[j] : a.k;
       const int64_t diff = ref - tok;
@@ -311,6 +333,7 @@ __global__ void __launch_bounds__(SCAN_THREADS, GBA_SCAN_MINB)
         const bool done = s_done != 0;
         __syncthreads();  // the shared words are rewritten by the next round
         if (done) break;
+        if (take == 0u && GBA_LOOKBACK_SLEEP_NS > 0) __nanosleep(GBA_LOOKBACK_SLEEP_NS);  // back off while predecessors work
         j -= take;
       }
       if (tid == 0)
@@ -473,16 +496,105 @@ __device__ __forceinline__ RowMeta row_meta(const SegOut& so, uint32_t u, uint32
   return r;
 }
 
-// Long rows go to the warp-per-chunk kernel: record the row, list its chunks,
-// and reserve chunk-sum slots when it has more than one chunk.
-__device__ __forceinline__ void hand_off_long_row(const SegOut& so, uint32_t u, const RowMeta& r) {
-  const uint32_t nch = (r.n + LONG_CHUNK - 1) / LONG_CHUNK;
-  const uint32_t li = atomicAdd(so.n_long, 1u);
-  const uint32_t base = atomicAdd(so.n_items, nch);
-  const uint32_t pb = nch > 1u ? atomicAdd(so.n_parts, nch) : 0u;
-  so.long_rows[li] = make_uint4(u, r.ks, r.n, pb);
-  so.long_done[li] = 0u;
-  for (uint32_t c = 0; c < nch; ++c) so.items[base + c] = make_uint2(li, c);
+// ---------------------------------------------------------------------------
+// k_row_classify: lists the rows with more than LONG_ROW kept occurrences for
+// the long-row kernel.  With small_ok, rows of at most SMALL_MAX kept
+// occurrences go to a list of their own (row, first kept entry, count,
+// denominator), each applied there by one lane group; longer rows are listed
+// with their chunks of LONG_CHUNK, each chunk summed by one warp.  Tiles of
+// 2048 row records (8 per thread); a block reserves a tile's entries with one
+// atomic per counter.  The order of the lists depends on the atomics, the
+// results do not: every row's chunks are summed and merged in chunk order.
+// ---------------------------------------------------------------------------
+constexpr int CLS_THREADS = 256, CLS_ITEMS = 8;  // rows per tile: 2048
+
+__global__ void __launch_bounds__(CLS_THREADS)
+    k_row_classify(StepArgs a, SegOut so, ErrSink err, int small_ok) {
+  __shared__ uint32_t s_w[4][CLS_THREADS / 32];
+  __shared__ uint32_t s_b[4];
+  if (__syncthreads_or(ld_volatile_u32(err.step) != 0u)) return;
+  const uint32_t U = ld_volatile_u32(so.total);
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t small_max = small_ok ? (uint32_t)SMALL_MAX : (uint32_t)LONG_ROW;
+  const uint32_t tile_rows = CLS_THREADS * CLS_ITEMS;
+  for (uint32_t t0 = blockIdx.x * tile_rows; t0 < U; t0 += gridDim.x * tile_rows) {
+    // this thread's rows t0 + tid*8 .. +7: kind and sizes
+    const uint32_t u0 = t0 + (uint32_t)tid * CLS_ITEMS;
+    uint32_t n_[CLS_ITEMS];
+    uint32_t cnt[4] = {0u, 0u, 0u, 0u};  // small rows, long rows, chunks, chunk-sum slots
+    uint4 prev = u0 < U ? so.rr[u0] : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+    for (int k = 0; k < CLS_ITEMS; ++k) {
+      const uint32_t u = u0 + k;
+      n_[k] = 0u;
+      if (u < U) {
+        const uint4 nx = so.rr[u + 1];
+        n_[k] = nx.y - prev.y;
+        prev = nx;
+      }
+      const uint32_t n = n_[k];
+      if (n > (uint32_t)LONG_ROW && n <= small_max) {
+        ++cnt[0];
+      } else if (n > small_max) {
+        const uint32_t nch = (n + LONG_CHUNK - 1) / LONG_CHUNK;
+        ++cnt[1];
+        cnt[2] += nch;
+        cnt[3] += nch > 1u ? nch : 0u;
+      }
+    }
+    // block-wide exclusive scans of the four counters; one atomic per counter
+    uint32_t excl[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      uint32_t v = cnt[c];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(FULL, v, o);
+        if (lane >= o) v += y;
+      }
+      excl[c] = v - cnt[c];
+      if (lane == 31) s_w[c][warp] = v;
+    }
+    __syncthreads();
+    if (tid < 4) {
+      uint32_t tot = 0u;
+      for (int w = 0; w < CLS_THREADS / 32; ++w) tot += s_w[tid][w];
+      uint32_t* ctr = tid == 0 ? so.n_small : (tid == 1 ? so.n_long : (tid == 2 ? so.n_items : so.n_parts));
+      s_b[tid] = tot ? atomicAdd(ctr, tot) : 0u;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      uint32_t before = 0u;
+      for (int w = 0; w < warp; ++w) before += s_w[c][w];
+      excl[c] += before + s_b[c];
+    }
+    if (cnt[0] | cnt[1]) {
+      prev = so.rr[u0];
+#pragma unroll
+      for (int k = 0; k < CLS_ITEMS; ++k) {
+        const uint32_t u = u0 + k;
+        const uint32_t n = n_[k];
+        if (u >= U) break;
+        const uint4 nx = so.rr[u + 1];
+        if (n > (uint32_t)LONG_ROW && n <= small_max) {
+          so.small_rows[excl[0]++] = make_uint4(
+              prev.x, prev.y, n,
+              __float_as_uint(row_denominator(a.sparse_den, nx.z - prev.z, nx.w - prev.w, a.M)));
+        } else if (n > small_max) {
+          const uint32_t nch = (n + LONG_CHUNK - 1) / LONG_CHUNK;
+          const uint32_t li = excl[1]++;
+          so.long_rows[li] = make_uint4(u, prev.y, n, nch > 1u ? excl[3] : 0u);
+          so.long_done[li] = 0u;
+          for (uint32_t c = 0; c < nch; ++c) so.items[excl[2] + c] = make_uint2(li, c);
+          excl[2] += nch;
+          excl[3] += nch > 1u ? nch : 0u;
+        }
+        prev = nx;
+      }
+    }
+    __syncthreads();  // s_w and s_b are rewritten by the next tile
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -506,6 +618,7 @@ __global__ void __launch_bounds__(ROW_THREADS, (CH * CPL <= 4) ? 3 : 2)
   const int64_t gw = (int64_t)blockIdx.x * (ROW_THREADS / 32) + (threadIdx.x >> 5);
   const int64_t TG = (int64_t)gridDim.x * (ROW_THREADS / 32) * G;
   const bool adam = tb.opt.kind == 1;
+  const bool unit = a.decay == 0;  // every kept weight is 1
   const int mode = a.sparse_den;
   const int32_t tag = (int32_t)(a.k + 1);
   uint32_t applied = 0u;
@@ -533,7 +646,6 @@ __global__ void __launch_bounds__(ROW_THREADS, (CH * CPL <= 4) ? 3 : 2)
     }
     // ---- this row: state and gradients, then the sums in sorted order
     const bool active = u < (int64_t)U && cur.n > 0u && cur.n <= (uint32_t)LONG_ROW;
-    if (u < (int64_t)U && cur.n > (uint32_t)LONG_ROW && l == 0) hand_off_long_row(so, (uint32_t)u, cur);
     Part<CH, CPL> w, s0, s1;
     if (active) {
       const size_t base = (size_t)cur.x * (size_t)d;
@@ -571,7 +683,7 @@ __global__ void __launch_bounds__(ROW_THREADS, (CH * CPL <= 4) ? 3 : 2)
           for (int c = 0; c < CPL; ++c) {
             if (l + c * L >= C) continue;
 #pragma unroll
-            for (int k = 0; k < CH; ++k) csum_add_prod(acc[c * CH + k], fw[e], gr[e].v[c * CH + k]);
+            for (int k = 0; k < CH; ++k) csum_add_w(acc[c * CH + k], unit, fw[e], gr[e].v[c * CH + k]);
           }
         }
       }
@@ -605,8 +717,8 @@ __global__ void __launch_bounds__(ROW_THREADS, (CH * CPL <= 4) ? 3 : 2)
 #ifndef GBA_STAGE_P
 #define GBA_STAGE_P 2
 #endif
-#ifndef GBA_STAGE_WIDE
-#define GBA_STAGE_WIDE 0
+#ifndef GBA_STAGE_CPL
+#define GBA_STAGE_CPL 1  // 16-byte pieces per lane for rows of up to 128 floats
 #endif
 constexpr int STAGE_P = GBA_STAGE_P;  // rows in flight per lane group
 constexpr int STAGE_NG = LONG_ROW;  // every kept gradient row of a row applied here is staged
@@ -645,7 +757,7 @@ __host__ __device__ constexpr int stage_floats_per_warp(int CPL, int regions, in
 #define GBA_STAGE_MINB 6
 #endif
 template <int CPL>
-__global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : 4)
+__global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : (CPL == 2 ? 4 : 2))
     k_row_apply_staged(StepArgs a, SegTable tb, SegOut so, DevStats* st, ErrSink err) {
   extern __shared__ __align__(16) float s_stage[];
   if (__any_sync(FULL, ld_volatile_u32(err.step) != 0u)) return;
@@ -661,6 +773,7 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : 4)
   const int64_t gw = (int64_t)blockIdx.x * (STAGE_THREADS / 32) + warp;
   const int64_t TG = (int64_t)gridDim.x * (STAGE_THREADS / 32) * G;
   const bool adam = tb.opt.kind == 1;
+  const bool unit = a.decay == 0;  // every kept weight is 1
   const int NS = adam ? 3 : 2;
   const int RS = L * CPL * 4;  // floats per region of a data slot
   const int SL = STAGE_META + (NS + STAGE_NG) * RS;
@@ -719,7 +832,6 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : 4)
           make_float4(__uint_as_float(m.x), __uint_as_float(short_row ? m.n : 0u), m.den, 0.f);
       *reinterpret_cast<float4*>(sl + 4) = short_row ? *reinterpret_cast<const float4*>(k + 8)
                                                      : make_float4(0.f, 0.f, 0.f, 0.f);
-      if (live && m.n > (uint32_t)LONG_ROW) hand_off_long_row(so, (uint32_t)u, m);
     }
     if (short_row) {
       const size_t base = (size_t)m.x * (size_t)d;
@@ -800,7 +912,7 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : 4)
               const float4 gv = *reinterpret_cast<const float4*>(dq + (NS + e) * RS);
               const float gb[4] = {gv.x, gv.y, gv.z, gv.w};
 #pragma unroll
-              for (int k = 0; k < 4; ++k) csum_add_prod(acc[4 * c + k], f[e], gb[k]);
+              for (int k = 0; k < 4; ++k) csum_add_w(acc[4 * c + k], unit, f[e], gb[k]);
             }
           }
         }
@@ -831,6 +943,12 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : 4)
 #define GBA_LONG_UNROLL 4
 #endif
 constexpr int LONG_UNROLL = GBA_LONG_UNROLL;
+#ifndef GBA_LONG_BPS
+#define GBA_LONG_BPS 0  // blocks per SM of the long-row kernel (0: as many as fit)
+#endif
+#ifndef GBA_STAGE_BPS_CUT
+#define GBA_STAGE_BPS_CUT 0  // staged blocks per SM left free for other kernels
+#endif
 constexpr int LONG_SLOTS = 4;  // list entries per lane: a group's part is at most 4 L entries
 static_assert(LONG_CHUNK <= 32 * LONG_SLOTS, "a chunk's part must fit the lanes' slots");
 
@@ -850,6 +968,7 @@ __global__ void __launch_bounds__(ROW_THREADS)
   const int lane = threadIdx.x & 31;
   const int g = lane >> lg, l = lane & (L - 1);
   const bool adam = tb.opt.kind == 1;
+  const bool unit = a.decay == 0;  // every kept weight is 1
   uint32_t applied = 0u;
 
   // the warp's next item is claimed and its description loaded while the
@@ -908,7 +1027,7 @@ __global__ void __launch_bounds__(ROW_THREADS)
           for (int c = 0; c < CPL; ++c) {
             if (l + c * L >= C) continue;
 #pragma unroll
-            for (int k = 0; k < CH; ++k) csum_add_prod(acc[c * CH + k], fw[e], gr[e].v[c * CH + k]);
+            for (int k = 0; k < CH; ++k) csum_add_w(acc[c * CH + k], unit, fw[e], gr[e].v[c * CH + k]);
           }
         }
       }
@@ -984,6 +1103,290 @@ __global__ void __launch_bounds__(ROW_THREADS)
 }
 
 // ---------------------------------------------------------------------------
+// k_row_long_staged: the long rows for widths that are a multiple of 4, with
+// their gradient rows staged in shared memory by cp.async so that many rows
+// are in flight per warp.
+//  1. Chunks of rows with more than SMALL_MAX kept occurrences, one warp per
+//     chunk as in k_row_long; each lane group's part of the chunk streams
+//     through a double buffer of LUNR rows per group.
+//  2. Rows of LONG_ROW + 1 .. SMALL_MAX kept occurrences, one lane group per
+//     row: its list entries, then its state and every kept gradient row are
+//     copied at once; warps claim G rows at a time.
+// Sums run over the kept entries in list order (per lane group part, parts
+// merged in group order, chunks in chunk order), as in k_row_long.
+// ---------------------------------------------------------------------------
+#ifndef GBA_LUNR
+#define GBA_LUNR 16
+#endif
+constexpr int LUNR = GBA_LUNR;  // rows per lane group per buffer in part 1
+constexpr int LONG_STAGE_THREADS = 128;
+
+__host__ __device__ constexpr int long_group_floats(int L, int CPL) {
+  // list entries (SMALL_MAX addresses + weights), state (3 rows), gradient rows
+  return 3 * SMALL_MAX + (3 + SMALL_MAX) * L * 4 * CPL;
+}
+__host__ __device__ constexpr int long_warp_floats(int L, int CPL) {
+  return (2 * LUNR * 32 * 4 * CPL) > ((32 / L) * long_group_floats(L, CPL))
+             ? (2 * LUNR * 32 * 4 * CPL)
+             : ((32 / L) * long_group_floats(L, CPL));
+}
+
+template <int CPL>
+__global__ void __launch_bounds__(LONG_STAGE_THREADS)
+    k_row_long_staged(StepArgs a, SegTable tb, SegOut so, DevStats* st, ErrSink err) {
+  extern __shared__ __align__(16) float s_long[];
+  if (__any_sync(FULL, ld_volatile_u32(err.step) != 0u)) return;
+  const int d = tb.d;
+  const int C = d >> 2;
+  int L = 1;
+  while (L * CPL < C && L < 32) L <<= 1;
+  const int lg = __ffs(L) - 1;
+  const int G = 32 >> lg;  // lane groups per warp
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int g = lane >> lg, l = lane & (L - 1);
+  const bool adam = tb.opt.kind == 1;
+  const bool unit = a.decay == 0;  // every kept weight is 1
+  const int RS = L * 4 * CPL;      // floats of one row in shared memory
+  const int32_t tag = (int32_t)(a.k + 1);
+  float* wsm = s_long + (size_t)warp * long_warp_floats(L, CPL);
+  uint32_t applied = 0u;
+
+  // ---- 1. chunks of the longest rows, one warp per chunk
+  {
+    const uint32_t n_items = ld_volatile_u32(so.n_items);
+    const uint32_t U = ld_volatile_u32(so.total);
+    auto claim = [&]() {
+      uint32_t t = 0u;
+      if (lane == 0) t = atomicAdd(so.item_ticket, 1u);
+      return __shfl_sync(FULL, t, 0);
+    };
+    uint32_t it = claim();
+    uint2 item = it < n_items ? so.items[it] : make_uint2(0u, 0u);
+    uint4 lr = it < n_items ? so.long_rows[item.x] : make_uint4(0u, 0u, 0u, 0u);
+    while (it < n_items) {
+      const uint32_t it_next = claim();
+      const uint2 item_next = it_next < n_items ? so.items[it_next] : make_uint2(0u, 0u);
+      const uint32_t nch = (lr.z + LONG_CHUNK - 1) / LONG_CHUNK;
+      const uint32_t e0 = lr.y + item.y * LONG_CHUNK;
+      const uint32_t e1 = min(e0 + (uint32_t)LONG_CHUNK, lr.y + lr.z);
+      const uint32_t per = (e1 - e0 + G - 1) / G;
+      const uint32_t b0 = min(e0 + g * per, e1), b1 = min(b0 + per, e1);
+      const uint32_t mine = b1 - b0;
+      const float* ptr[LONG_SLOTS];
+      float wgt[LONG_SLOTS];
+#pragma unroll
+      for (int s2 = 0; s2 < LONG_SLOTS; ++s2) {
+        const uint32_t j = (uint32_t)(l + s2 * L);
+        ptr[s2] = j < mine ? so.kl[b0 + j] : nullptr;
+        wgt[s2] = j < mine ? so.kw[b0 + j] : 0.f;
+      }
+      uint32_t most = mine;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) most = max(most, __shfl_xor_sync(FULL, most, o));
+      CSum acc[4 * CPL];
+#pragma unroll
+      for (int i = 0; i < 4 * CPL; ++i) acc[i] = CSum{0.f, 0.f};
+      // entries j0 .. j0 + LUNR - 1 of every group's part into buffer bsel
+      auto stage = [&](uint32_t j0, int bsel) {
+#pragma unroll 4
+        for (int e = 0; e < LUNR; ++e) {
+          const uint32_t j = j0 + (uint32_t)e;
+          const uint32_t s2 = j >> lg;
+          const int src = (int)(j & (uint32_t)(L - 1));
+          const float* pj = s2 == 0 ? ptr[0] : (s2 == 1 ? ptr[1] : (s2 == 2 ? ptr[2] : ptr[3]));
+          pj = (const float*)__shfl_sync(FULL, (unsigned long long)pj, src, L);
+          if (j < mine) {
+            float* dst = wsm + ((size_t)(bsel * G + g) * LUNR + e) * RS;
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+              const int q = l + c * L;
+              if (q < C) cp_async16(dst + 4 * q, pj + 4 * q);
+            }
+          }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+      };
+      stage(0u, 0);
+      int bsel = 0;
+      for (uint32_t j0 = 0; j0 < most; j0 += LUNR, bsel ^= 1) {
+        if (j0 + LUNR < most) {
+          stage(j0 + LUNR, bsel ^ 1);
+          asm volatile("cp.async.wait_group 1;" ::: "memory");
+        } else {
+          asm volatile("cp.async.wait_group 0;" ::: "memory");
+        }
+        __syncwarp();
+        for (int e = 0; e < LUNR; ++e) {
+          const uint32_t j = j0 + (uint32_t)e;
+          const uint32_t s2 = j >> lg;
+          const int src = (int)(j & (uint32_t)(L - 1));
+          float wj = s2 == 0 ? wgt[0] : (s2 == 1 ? wgt[1] : (s2 == 2 ? wgt[2] : wgt[3]));
+          wj = __shfl_sync(FULL, wj, src, L);
+          if (j < mine) {
+            const float* rowp = wsm + ((size_t)(bsel * G + g) * LUNR + e) * RS;
+#pragma unroll
+            for (int c = 0; c < CPL; ++c) {
+              const int q = l + c * L;
+              if (q >= C) continue;
+              const float4 v = *reinterpret_cast<const float4*>(rowp + 4 * q);
+              csum_add_w(acc[4 * c + 0], unit, wj, v.x);
+              csum_add_w(acc[4 * c + 1], unit, wj, v.y);
+              csum_add_w(acc[4 * c + 2], unit, wj, v.z);
+              csum_add_w(acc[4 * c + 3], unit, wj, v.w);
+            }
+          }
+        }
+        __syncwarp();  // the buffer is refilled next
+      }
+      // the groups' parts in group order, into group 0
+      for (int gg = 1; gg < G; ++gg) {
+#pragma unroll
+        for (int i = 0; i < 4 * CPL; ++i) {
+          const float hi = __shfl_sync(FULL, acc[i].hi, gg * L + l);
+          const float lo = __shfl_sync(FULL, acc[i].lo, gg * L + l);
+          if (g == 0) csum_merge(acc[i], hi, lo);
+        }
+      }
+      bool finish = nch == 1u;
+      if (!finish) {  // one chunk of several: leave its sum; the last chunk finishes the row
+        if (g == 0) {
+          const size_t pb = (size_t)(lr.w + item.y) * (size_t)so.pstride;
+#pragma unroll
+          for (int c = 0; c < CPL; ++c)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const int q = l + c * L;
+              if (q < C) {
+                so.part_hi[pb + (size_t)q * 4 + k] = acc[c * 4 + k].hi;
+                so.part_lo[pb + (size_t)q * 4 + k] = acc[c * 4 + k].lo;
+              }
+            }
+        }
+        __threadfence();
+        __syncwarp();
+        uint32_t last = 0u;
+        if (lane == 0) last = atomicAdd(so.long_done + item.x, 1u) == nch - 1u;
+        finish = __shfl_sync(FULL, last, 0) != 0u;
+        if (finish) {  // every chunk's sum is visible: merge them in chunk order
+          __threadfence();
+#pragma unroll
+          for (int i = 0; i < 4 * CPL; ++i) acc[i] = CSum{0.f, 0.f};
+          for (uint32_t cc = 0; cc < nch; ++cc) {
+            const size_t qb = (size_t)(lr.w + cc) * (size_t)so.pstride;
+#pragma unroll
+            for (int c = 0; c < CPL; ++c)
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const int q = l + c * L;
+                if (q < C && g == 0)
+                  csum_merge(acc[c * 4 + k], __ldcg(so.part_hi + qb + (size_t)q * 4 + k),
+                             __ldcg(so.part_lo + qb + (size_t)q * 4 + k));
+              }
+          }
+        }
+      }
+      if (finish && g == 0) {
+        const RowMeta r = row_meta(so, lr.x, U, a.sparse_den, a.M);
+        Part<4, CPL> w, s0, s1;
+        const size_t base = (size_t)r.x * (size_t)d;
+        load_part<4, CPL>(tb.w + base, l, L, C, w);
+        load_part<4, CPL>(tb.s0 + base, l, L, C, s0);
+        if (adam) load_part<4, CPL>(tb.s1 + base, l, L, C, s1);
+        finish_row<4, CPL>(tb, r.x, r.den, acc, w, s0, s1, l, L, C, adam);
+        if (l == 0) {
+          tb.ver[r.x] = tag;
+          ++applied;
+        }
+      }
+      __syncwarp();
+      it = it_next;
+      item = item_next;
+      lr = it < n_items ? so.long_rows[item.x] : make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+
+  // ---- 2. rows of LONG_ROW + 1 .. SMALL_MAX kept occurrences, one lane group each
+  {
+    const uint32_t n_small = ld_volatile_u32(so.n_small);
+    const int GF = long_group_floats(L, CPL);
+    float* gs = wsm + (size_t)g * GF;
+    const float** pp = reinterpret_cast<const float**>(gs);  // [SMALL_MAX] addresses
+    float* wt = gs + 2 * SMALL_MAX;                           // [SMALL_MAX] weights
+    float* sst = gs + 3 * SMALL_MAX;                          // w, s0, s1
+    float* rows = sst + 3 * RS;                               // [SMALL_MAX] gradient rows
+    auto claim = [&]() {
+      uint32_t t = 0u;
+      if (lane == 0) t = atomicAdd(so.small_ticket, (uint32_t)G);
+      return __shfl_sync(FULL, t, 0);
+    };
+    uint32_t base = claim();
+    uint4 sr = base + g < n_small ? so.small_rows[base + g] : make_uint4(0u, 0u, 0u, 0u);
+    while (base < n_small) {
+      const uint32_t x = sr.x, ks = sr.y, n = sr.z;  // n = 0: no row for this group
+      for (uint32_t e = (uint32_t)l; e < n; e += (uint32_t)L) {
+        cp_async8(pp + e, so.kl + ks + e);
+        cp_async4(wt + e, so.kw + ks + e);
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+      __syncwarp();
+      if (n > 0u) {
+        const size_t rb = (size_t)x * (size_t)d;
+#pragma unroll
+        for (int c = 0; c < CPL; ++c) {
+          const int q = l + c * L;
+          if (q >= C) continue;
+          cp_async16(sst + 4 * q, tb.w + rb + 4 * q);
+          cp_async16(sst + RS + 4 * q, tb.s0 + rb + 4 * q);
+          if (adam) cp_async16(sst + 2 * RS + 4 * q, tb.s1 + rb + 4 * q);
+          for (uint32_t e = 0; e < n; ++e) cp_async16(rows + (size_t)e * RS + 4 * q, pp[e] + 4 * q);
+        }
+      }
+      asm volatile("cp.async.commit_group;" ::: "memory");
+      // the next rows are claimed while these land
+      const uint32_t base_next = claim();
+      const uint4 sr_next =
+          base_next + g < n_small ? so.small_rows[base_next + g] : make_uint4(0u, 0u, 0u, 0u);
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+      __syncwarp();
+      if (n > 0u) {
+        CSum acc[4 * CPL];
+#pragma unroll
+        for (int i = 0; i < 4 * CPL; ++i) acc[i] = CSum{0.f, 0.f};
+        for (uint32_t e = 0; e < n; ++e) {
+          const float we = wt[e];
+#pragma unroll
+          for (int c = 0; c < CPL; ++c) {
+            const int q = l + c * L;
+            if (q >= C) continue;
+            const float4 v = *reinterpret_cast<const float4*>(rows + (size_t)e * RS + 4 * q);
+            csum_add_w(acc[4 * c + 0], unit, we, v.x);
+            csum_add_w(acc[4 * c + 1], unit, we, v.y);
+            csum_add_w(acc[4 * c + 2], unit, we, v.z);
+            csum_add_w(acc[4 * c + 3], unit, we, v.w);
+          }
+        }
+        Part<4, CPL> w, s0, s1;
+        load_part<4, CPL>(sst, l, L, C, w);
+        load_part<4, CPL>(sst + RS, l, L, C, s0);
+        if (adam) load_part<4, CPL>(sst + 2 * RS, l, L, C, s1);
+        finish_row<4, CPL>(tb, x, __uint_as_float(sr.w), acc, w, s0, s1, l, L, C, adam);
+        if (l == 0) {
+          tb.ver[x] = tag;
+          ++applied;
+        }
+      }
+      __syncwarp();  // every lane is done with the group's buffers
+      base = base_next;
+      sr = sr_next;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) applied += __shfl_xor_sync(FULL, applied, o);
+  if (lane == 0 && applied) atomicAdd(&st->rows_applied, (unsigned long long)applied);
+}
+
+// ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
 template <typename K>
@@ -1010,7 +1413,8 @@ void launch_staged(const StepArgs& a, const SegTable& tb, const SegOut& so, DevS
       cudaFuncSetAttribute(k_row_apply_staged<CPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem_max) == cudaSuccess;
   (void)configured;
-  const int bps = blocks_per_sm(k_row_apply_staged<CPL>, STAGE_THREADS, smem);
+  const int bps = std::max(1, blocks_per_sm(k_row_apply_staged<CPL>, STAGE_THREADS, smem) -
+                                 GBA_STAGE_BPS_CUT);
   const int64_t Nt = tb.pos_end - tb.pos_begin;  // bounds the rows
   const int64_t rows_per_block = (int64_t)(STAGE_THREADS / 32) * G * STAGE_P;
   const int64_t grid = std::max<int64_t>(
@@ -1022,7 +1426,10 @@ template <int CH, int CPL>
 void launch_apply_cfg(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
                       ErrSink err, int num_sms, cudaStream_t s) {
   if constexpr (CH == 4) {
-    launch_staged<GBA_STAGE_WIDE ? 2 : CPL>(a, tb, so, stats, err, num_sms, s);
+    if (CPL == 1 && GBA_STAGE_CPL != 1 && tb.d >= 32)  // wider pieces per lane for wide rows
+      launch_staged<GBA_STAGE_CPL>(a, tb, so, stats, err, num_sms, s);
+    else
+      launch_staged<CPL>(a, tb, so, stats, err, num_sms, s);
     return;
   }
   static const int bps = blocks_per_sm(k_row_apply<CH, CPL>, ROW_THREADS, 0);
@@ -1036,10 +1443,38 @@ void launch_apply_cfg(const StepArgs& a, const SegTable& tb, const SegOut& so, D
   k_row_apply<CH, CPL><<<(unsigned)grid, ROW_THREADS, 0, s>>>(a, tb, so, stats, err);
 }
 
+template <int CPL>
+void launch_long_staged(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
+                        ErrSink err, int num_sms, cudaStream_t s) {
+  const int C = tb.d / 4;
+  int L = 1;
+  while (L * CPL < C && L < 32) L <<= 1;
+  const size_t smem = (size_t)(LONG_STAGE_THREADS / 32) * long_warp_floats(L, CPL) * 4;
+  static size_t attr = 0;  // the largest dynamic shared memory size set so far
+  if (smem > attr &&
+      cudaFuncSetAttribute(k_row_long_staged<CPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) == cudaSuccess)
+    attr = smem;
+  const int bps = GBA_LONG_BPS > 0
+                      ? GBA_LONG_BPS
+                      : blocks_per_sm(k_row_long_staged<CPL>, LONG_STAGE_THREADS, smem);
+  const int64_t Nt = tb.pos_end - tb.pos_begin;
+  const int64_t max_items = Nt / (LONG_ROW + 1) + Nt / LONG_CHUNK + 1;
+  const int64_t grid = std::max<int64_t>(
+      1, std::min<int64_t>((int64_t)num_sms * bps,
+                           (max_items + LONG_STAGE_THREADS / 32 - 1) / (LONG_STAGE_THREADS / 32)));
+  k_row_long_staged<CPL><<<(unsigned)grid, LONG_STAGE_THREADS, smem, s>>>(a, tb, so, stats, err);
+}
+
 template <int CH, int CPL>
 void launch_long_cfg(const StepArgs& a, const SegTable& tb, const SegOut& so, DevStats* stats,
                      ErrSink err, int num_sms, cudaStream_t s) {
-  static const int bps = blocks_per_sm(k_row_long<CH, CPL>, ROW_THREADS, 0);
+  if constexpr (CH == 4) {
+    launch_long_staged<CPL>(a, tb, so, stats, err, num_sms, s);
+    return;
+  }
+  static const int bps = GBA_LONG_BPS > 0 ? GBA_LONG_BPS
+                                         : blocks_per_sm(k_row_long<CH, CPL>, ROW_THREADS, 0);
   const int64_t Nt = tb.pos_end - tb.pos_begin;
   const int64_t max_items = Nt / (LONG_ROW + 1) + Nt / LONG_CHUNK + 1;
   const int64_t grid = std::max<int64_t>(
@@ -1050,6 +1485,16 @@ void launch_long_cfg(const StepArgs& a, const SegTable& tb, const SegOut& so, De
 }  // namespace
 
 int64_t scan_tiles(int64_t N) { return (N + SCAN_TILE - 1) / SCAN_TILE; }
+
+void launch_row_classify(const StepArgs& a, const SegTable& tb, const SegOut& so, ErrSink err,
+                         int num_sms, cudaStream_t s) {
+  const int64_t Nt = tb.pos_end - tb.pos_begin;  // bounds the rows
+  const int64_t tile_rows = CLS_THREADS * CLS_ITEMS;
+  const int64_t grid =
+      std::max<int64_t>(1, std::min<int64_t>((int64_t)num_sms * 4, (Nt + tile_rows - 1) / tile_rows));
+  // widths that are a multiple of 4 use the staged long-row kernel and its list of small rows
+  k_row_classify<<<(unsigned)grid, CLS_THREADS, 0, s>>>(a, so, err, (tb.d & 3) == 0 ? 1 : 0);
+}
 
 void launch_seg_scan(const StepArgs& a, const SegTable& tb, const SegOut& so, const uint32_t* keys,
                      const uint32_t* vals, DevStats* stats, ErrSink err, int64_t wait_ns,

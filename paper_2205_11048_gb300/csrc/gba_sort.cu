@@ -211,6 +211,9 @@ __global__ void __launch_bounds__(SORT_THREADS) k_sort_histogram(StepArgs a, int
 // ---------------------------------------------------------------------------
 // One onesweep pass over 8 bits of the key.
 // ---------------------------------------------------------------------------
+#ifndef GBA_LOOKBACK_SLEEP_NS
+#define GBA_LOOKBACK_SLEEP_NS 64
+#endif
 template <bool FIRST>
 __global__ void __launch_bounds__(SORT_THREADS)
     k_onesweep(StepArgs a, int pass, const uint32_t* __restrict__ keys_in,
@@ -320,10 +323,13 @@ __global__ void __launch_bounds__(SORT_THREADS)
       if (done) break;
       j -= used;
       if (j < 0) break;  // cannot happen: tile 0 publishes an inclusive prefix
-      if (used == 0 && ((ld_volatile_u32(err.step) & ERR_TIMEOUT) ||
-                        (int64_t)(globaltimer_ns() - t0) > wait_ns)) {
-        raise_error(err, ERR_TIMEOUT);
-        break;
+      if (used == 0) {
+        if ((ld_volatile_u32(err.step) & ERR_TIMEOUT) ||
+            (int64_t)(globaltimer_ns() - t0) > wait_ns) {
+          raise_error(err, ERR_TIMEOUT);
+          break;
+        }
+        if (GBA_LOOKBACK_SLEEP_NS > 0) __nanosleep(GBA_LOOKBACK_SLEEP_NS);  // back off: spinning takes issue slots from the tiles it waits for
       }
     }
     st_relaxed_u64(my, ep | FLAG_INCL | ((prefix + tile_count) & COUNT_MASK));
