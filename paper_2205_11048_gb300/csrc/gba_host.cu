@@ -82,8 +82,8 @@ size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 
 }  // namespace
 
-#ifndef GBA_LONG_STREAM
-#define GBA_LONG_STREAM 0
+#ifndef GBA_STREAM_PRIO
+#define GBA_STREAM_PRIO 0
 #endif
 
 struct gba_handle {
@@ -94,8 +94,6 @@ struct gba_handle {
   cudaStream_t side = nullptr;   // dense update
   cudaStream_t sorts = nullptr;   // message weights, histogram, sort passes
   cudaStream_t applys = nullptr;  // segment-sum and row update
-  cudaStream_t longs = nullptr;   // long rows (when run beside the short rows)
-  cudaEvent_t ev_classified = nullptr, ev_longs = nullptr;
   bool overlap = false;           // consecutive steps may run concurrently
   cudaEvent_t ev_pushes = nullptr;
   cudaEvent_t ev_hist[SLOTS] = {}, ev_sorted[SLOTS] = {}, ev_applied[SLOTS] = {},
@@ -295,7 +293,6 @@ void free_all(gba_handle* h) {
   cudaSetDevice(h->device);
   if (h->sorts) cudaStreamSynchronize(h->sorts);
   if (h->applys) cudaStreamSynchronize(h->applys);
-  if (h->longs) cudaStreamSynchronize(h->longs);
   if (h->side) cudaStreamSynchronize(h->side);
   if (h->stream) cudaStreamSynchronize(h->stream);
   for (auto& t : h->tables) {
@@ -348,9 +345,6 @@ void free_all(gba_handle* h) {
   }
   for (auto e : h->event_pool) cudaEventDestroy(e);
   if (h->ev_pushes) cudaEventDestroy(h->ev_pushes);
-  if (h->ev_classified) cudaEventDestroy(h->ev_classified);
-  if (h->ev_longs) cudaEventDestroy(h->ev_longs);
-  if (h->longs) cudaStreamDestroy(h->longs);
   if (h->side) cudaStreamDestroy(h->side);
   if (h->sorts) cudaStreamDestroy(h->sorts);
   if (h->applys) cudaStreamDestroy(h->applys);
@@ -358,9 +352,8 @@ void free_all(gba_handle* h) {
 }
 
 cudaError_t sync_all(gba_handle* h) {
-  cudaError_t e[5] = {cudaStreamSynchronize(h->sorts), cudaStreamSynchronize(h->applys),
-                      cudaStreamSynchronize(h->longs), cudaStreamSynchronize(h->side),
-                      cudaStreamSynchronize(h->stream)};
+  cudaError_t e[4] = {cudaStreamSynchronize(h->sorts), cudaStreamSynchronize(h->applys),
+                      cudaStreamSynchronize(h->side), cudaStreamSynchronize(h->stream)};
   for (cudaError_t x : e)
     if (x != cudaSuccess) return x;
   return cudaSuccess;
@@ -786,13 +779,18 @@ gba_status gba_create(const gba_table_desc* tables, int32_t n_tables, int64_t de
       return fail(GBA_E_CUDA);
     h->own_stream = true;
   }
-  if (cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&h->sorts, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&h->applys, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaStreamCreateWithFlags(&h->longs, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_pushes, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_classified, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&h->ev_longs, cudaEventDisableTiming) != cudaSuccess)
+  // Stream priorities (GBA_STREAM_PRIO): 0 all equal; 1 the row path first and
+  // the next step's sort last; 2 the row path first, the others equal.
+  int prio_lo = 0, prio_hi = 0;
+  if (GBA_STREAM_PRIO != 0 && cudaDeviceGetStreamPriorityRange(&prio_lo, &prio_hi) != cudaSuccess)
+    prio_lo = prio_hi = 0;
+  const int p_rows = GBA_STREAM_PRIO != 0 ? prio_hi : 0;
+  const int p_sort = GBA_STREAM_PRIO == 1 ? prio_lo : (GBA_STREAM_PRIO == 2 ? (prio_lo + prio_hi) / 2 : 0);
+  const int p_side = GBA_STREAM_PRIO != 0 ? (prio_lo + prio_hi) / 2 : 0;
+  if (cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, p_side) != cudaSuccess ||
+      cudaStreamCreateWithPriority(&h->sorts, cudaStreamNonBlocking, p_sort) != cudaSuccess ||
+      cudaStreamCreateWithPriority(&h->applys, cudaStreamNonBlocking, p_rows) != cudaSuccess ||
+      cudaEventCreateWithFlags(&h->ev_pushes, cudaEventDisableTiming) != cudaSuccess)
     return fail(GBA_E_CUDA);
   for (int b = 0; b < SLOTS; ++b)
     for (cudaEvent_t* e : {&h->ev_hist[b], &h->ev_sorted[b], &h->ev_applied[b], &h->ev_densed[b]})
@@ -1163,21 +1161,6 @@ int32_t gba_try_apply(gba_handle* h) {
         Timed tm(h, GBA_K_SEG_SCAN, h->applys);
         launch_row_classify(a, tb, so, sink, h->num_sms, h->applys);
       }
-#if GBA_LONG_STREAM
-      // long rows on their own stream, next to the short rows
-      cudaEventRecord(h->ev_classified, h->applys);
-      cudaStreamWaitEvent(h->longs, h->ev_classified, 0);
-      {
-        Timed tm(h, GBA_K_ROW_LONG, h->longs);
-        launch_row_long(a, tb, so, h->d_stats, sink, h->num_sms, h->longs);
-      }
-      {
-        Timed tm(h, GBA_K_ROW_APPLY, h->applys);
-        launch_row_apply(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
-      }
-      cudaEventRecord(h->ev_longs, h->longs);
-      cudaStreamWaitEvent(h->applys, h->ev_longs, 0);
-#else
       {
         Timed tm(h, GBA_K_ROW_APPLY, h->applys);
         launch_row_apply(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
@@ -1186,7 +1169,6 @@ int32_t gba_try_apply(gba_handle* h) {
         Timed tm(h, GBA_K_ROW_LONG, h->applys);
         launch_row_long(a, tb, so, h->d_stats, sink, h->num_sms, h->applys);
       }
-#endif
     }
   }
   if (N == 0) {

@@ -342,7 +342,10 @@ void launch_weights(const StepArgs& a, StepScratch sc, DevStats* stats, int n_hi
                     cudaStream_t s);
 
 // Keys per onesweep tile (also sizes the look-back words of the static sort).
-constexpr int SORT_TILE_KEYS = 2048;
+#ifndef GBA_SORT_TILE
+#define GBA_SORT_TILE 2048
+#endif
+constexpr int SORT_TILE_KEYS = GBA_SORT_TILE;  // keys per onesweep tile
 
 // Digit histograms of every pass; writes each occurrence's key to keys0 (the
 // first onesweep pass's input).

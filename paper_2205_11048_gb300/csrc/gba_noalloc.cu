@@ -47,7 +47,11 @@ constexpr size_t kOffTinfo = kOffNbase + 16;
 constexpr size_t kOffErr = kOffTinfo + 32;  // TableInfo is 24 bytes
 static_assert(sizeof(gba::TableInfo) <= 32, "TableInfo outgrew its scratch slot");
 constexpr size_t kBytes = kOffErr + 16;
+#if GBA_SORT_TILE == 2048
 static_assert(kBytes == GBA_STATIC_SORT_BYTES, "scratch size differs from the header");
+#else
+static_assert(kBytes <= GBA_STATIC_SORT_BYTES, "scratch larger than the header's size");
+#endif
 
 static __device__ __align__(256) unsigned char g_sort_scratch[kBytes];
 
