@@ -289,9 +289,9 @@ gba_status gba_lookup_rows(gba_handle* h, int32_t t, const int64_t* ids, int64_t
 /*
  * gba_set_eager_dense - when on, a pushed message's dense gradient is added to
  * the compensated sum of the global step it belongs to at push time, instead
- * of being kept until that step (the memory saving of the paper's Alg. 2
- * discussion: the weighted sum over some gradients can be executed in
- * advance, based on the tokens).  The FIFO fixes each message's step (the
+ * of being kept until that step (the memory saving that the discussion of
+ * Alg. 2 points out: the tokens fix the weights, so part of the weighted sum
+ * may be formed before the step).  The FIFO fixes each message's step (the
  * shortest prefix of buffered local batches reaching G), so its weight
  * (Eq. (1) or the decay strategy) is known when it arrives.  Sums are formed
  * in arrival order, the order of the buffered mode, so results are identical.

@@ -196,8 +196,8 @@ __global__ void __launch_bounds__(DENSE_THREADS)
 }
 
 // ---------------------------------------------------------------------------
-// Eager aggregation (Alg. 2 discussion: the weighted sum of the gradients can
-// be executed in advance, based on the tokens).  Under the FIFO every pushed
+// Eager aggregation (Alg. 2 discussion: because the tokens fix the weights,
+// part of the weighted sum may be formed before the step).  Under the FIFO every pushed
 // message belongs to a known future step, so its weight is known at push: its
 // dense gradient is added to that step's compensated accumulator (hi, lo)
 // right away, in push order -- the order the buffered K5 sums in -- and the
