@@ -5,14 +5,14 @@
 // or Adam in place -- one pass over HBM: every kept gradient is read once, the
 // weights and optimizer state are read and written once.
 //
-// Each persistent CTA walks an equal contiguous share of the parameters in
-// tiles of up to DT.  A producer warp streams the tile's slice of every kept
-// message into a ring of shared-memory stages with 1-D bulk async copies
-// (cp.async.bulk, completion counted on an mbarrier per stage); eight consumer
-// warps sum the slices with compensated (TwoSum) float arithmetic, release each
-// stage on an "empty" mbarrier, and finish the tile with the optimizer.  Every mbarrier wait is bounded in time; a wait that
-// gives up latches ERR_TIMEOUT, the CTA stops issuing copies, waits (bounded)
-// for the copies it already issued, and exits.
+// Each persistent CTA walks every gridDim-th tile of DT parameters.  A
+// producer warp streams the tile's slice of every kept message into a ring of
+// shared-memory stages with 1-D bulk async copies (cp.async.bulk, completion
+// counted on an mbarrier per stage); eight consumer warps sum the slices with
+// compensated (TwoSum) float arithmetic, release each stage on an "empty"
+// mbarrier, and finish the tile with the optimizer.  Every mbarrier wait is
+// bounded in time; a wait that gives up latches ERR_TIMEOUT, the CTA stops
+// issuing copies, waits (bounded) for the copies it already issued, and exits.
 #include "gba_internal.cuh"
 
 namespace gba {
@@ -57,19 +57,19 @@ __global__ void __launch_bounds__(DENSE_THREADS)
 
   const int n_kept = *sc.n_kept;
   const int64_t D4 = da.D & ~3ll;  // parameters streamed by bulk copies
-  // This CTA's contiguous range of parameters (equal shares, multiples of 4
-  // so every copy stays 16-byte aligned), walked in tiles of up to DT.
-  const int64_t q4 = D4 / 4;
-  const int64_t r0 = 4 * (q4 * (int64_t)blockIdx.x / gridDim.x);
-  const int64_t r1 = 4 * (q4 * ((int64_t)blockIdx.x + 1) / gridDim.x);
+  // This CTA's tiles of DT parameters (the last one shorter, a multiple of 4
+  // so every copy stays 16-byte aligned): blockIdx.x, blockIdx.x + gridDim.x,
+  // ...  At any moment the CTAs work on neighbouring tiles, so the copies from
+  // the kept messages' buffers touch few DRAM pages and TLB entries.
+  const int64_t t0 = (int64_t)blockIdx.x * DT, tstep = (int64_t)gridDim.x * DT;
 
   if (warp == CONSUMER_WARPS) {
     // ---- producer
     if (lane == 0) {
       uint32_t q = 0;
       bool ok = da.withhold == 0;
-      for (int64_t start = r0; start < r1 && ok; start += DT) {
-        const uint32_t bytes = (uint32_t)((r1 - start < DT ? r1 - start : DT) * sizeof(float));
+      for (int64_t start = t0; start < D4 && ok; start += tstep) {
+        const uint32_t bytes = (uint32_t)((D4 - start < DT ? D4 - start : DT) * sizeof(float));
         for (int j = 0; j < n_kept; ++j, ++q) {
           const int stage = (int)(q % STAGES);
           const uint32_t ph = (q / STAGES) & 1u;
@@ -99,8 +99,8 @@ __global__ void __launch_bounds__(DENSE_THREADS)
     const int c = tid;
     const float Mf = (float)da.M;
     uint32_t q = 0;
-    for (int64_t start = r0; start < r1; start += DT) {
-      const int64_t n = r1 - start < DT ? r1 - start : DT;
+    for (int64_t start = t0; start < D4; start += tstep) {
+      const int64_t n = D4 - start < DT ? D4 - start : DT;
       bool mine[PER];
       int64_t e[PER];
       float4 w[PER], s0[PER], s1[PER];

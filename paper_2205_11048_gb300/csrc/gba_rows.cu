@@ -725,9 +725,10 @@ constexpr int STAGE_NG = LONG_ROW;  // every kept gradient row of a row applied 
 constexpr int STAGE_META = 8;       // floats of row metadata at the head of a data slot
 constexpr int STAGE_THREADS = 128;
 // per lane group: records of 3P rows ahead (2 x 16 B each), list entries of
-// 2P rows ahead (4 addresses + 4 weights = 48 B each), P data slots
+// 2P rows ahead (4 addresses + 4 weights + the decoded record = 64 B each), P
+// data slots
 constexpr int STAGE_REC_FLOATS = 3 * STAGE_P * 8;
-constexpr int STAGE_KL_FLOATS = 2 * STAGE_P * 12;
+constexpr int STAGE_KL_FLOATS = 2 * STAGE_P * 16;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src)
@@ -770,8 +771,9 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : (CP
   const int G = 32 >> lg;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int g = lane >> lg, l = lane & (L - 1);
-  const int64_t gw = (int64_t)blockIdx.x * (STAGE_THREADS / 32) + warp;
-  const int64_t TG = (int64_t)gridDim.x * (STAGE_THREADS / 32) * G;
+  // row indices fit 32 bits (at most 2^30 occurrences per step)
+  const uint32_t gw = blockIdx.x * (uint32_t)(STAGE_THREADS / 32) + (uint32_t)warp;
+  const uint32_t TG = gridDim.x * (uint32_t)(STAGE_THREADS / 32) * (uint32_t)G;
   const bool adam = tb.opt.kind == 1;
   const bool unit = a.decay == 0;  // every kept weight is 1
   const int NS = adam ? 3 : 2;
@@ -779,26 +781,26 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : (CP
   const int SL = STAGE_META + (NS + STAGE_NG) * RS;
   float* wbase = s_stage + (size_t)warp * stage_floats_per_warp(CPL, NS + STAGE_NG, G);
   float* recs = wbase + (size_t)g * STAGE_REC_FLOATS;                       // [3P][8]
-  float* kls = wbase + (size_t)G * STAGE_REC_FLOATS + (size_t)g * STAGE_KL_FLOATS;  // [2P][12]
+  float* kls = wbase + (size_t)G * STAGE_REC_FLOATS + (size_t)g * STAGE_KL_FLOATS;  // [2P][16]
   float* data = wbase + (size_t)G * (STAGE_REC_FLOATS + STAGE_KL_FLOATS) + (size_t)g * STAGE_P * SL;
   const int mode = a.sparse_den;
   const int32_t tag = (int32_t)(a.k + 1);
   float* const state[3] = {tb.w, tb.s0, tb.s1};
   uint32_t applied = 0u;
-  const int64_t u0 = gw * G + g;
+  const uint32_t u0 = gw * (uint32_t)G + (uint32_t)g;
 
   // level A: the records of row i (two 16-byte words), or an empty record
-  auto level_a = [&](int64_t i) {
-    const int64_t u = u0 + i * TG;
+  auto level_a = [&](uint32_t i) {
+    const uint32_t u = u0 + i * TG;
     uint4* r = reinterpret_cast<uint4*>(recs + (size_t)(i % (3 * STAGE_P)) * 8);
-    if (u < (int64_t)U) {
+    if (u < U) {
       for (int e = l; e < 2; e += L) cp_async16(r + e, so.rr + u + e);  // L may be 1
     } else if (l == 0) {
       r[0] = make_uint4(0u, 0u, 0u, 0u);
       r[1] = make_uint4(0u, 0u, 0u, 0u);
     }
   };
-  auto decode = [&](int64_t i) {
+  auto decode = [&](uint32_t i) {
     const uint4* r = reinterpret_cast<const uint4*>(recs + (size_t)(i % (3 * STAGE_P)) * 8);
     const uint4 ra = r[0], rb = r[1];
     RowMeta m;
@@ -808,10 +810,14 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : (CP
     m.den = row_denominator(mode, rb.z - ra.z, rb.w - ra.w, a.M);
     return m;
   };
-  // level B: the kept entries of row i (addresses and weights)
-  auto level_b = [&](int64_t i) {
+  // level B: the kept entries of row i (addresses and weights); the decoded
+  // record is kept beside them for level C
+  auto level_b = [&](uint32_t i) {
     const RowMeta m = decode(i);
-    float* k = kls + (size_t)(i % (2 * STAGE_P)) * 12;
+    float* k = kls + (size_t)(i % (2 * STAGE_P)) * 16;
+    if (l == 0)
+      *reinterpret_cast<float4*>(k + 12) =
+          make_float4(__uint_as_float(m.x), __uint_as_float(m.n), m.den, 0.f);
     if (m.n > 0u && m.n <= (uint32_t)LONG_ROW) {
       for (uint32_t e = (uint32_t)l; e < m.n; e += (uint32_t)L) {  // L may be below LONG_ROW
         cp_async8(k + 2 * e, so.kl + m.ks + e);
@@ -820,12 +826,15 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : (CP
     }
   };
   // level C: weights, state and gradient rows of row i into data slot i % P
-  auto level_c = [&](int64_t i) {
-    const RowMeta m = decode(i);
-    const float* k = kls + (size_t)(i % (2 * STAGE_P)) * 12;
+  auto level_c = [&](uint32_t i) {
+    const float* k = kls + (size_t)(i % (2 * STAGE_P)) * 16;
+    const float4 km = *reinterpret_cast<const float4*>(k + 12);
+    RowMeta m;
+    m.x = __float_as_uint(km.x);
+    m.n = __float_as_uint(km.y);
+    m.den = km.z;
     float* sl = data + (size_t)(i % STAGE_P) * SL;
-    const int64_t u = u0 + i * TG;
-    const bool live = u < (int64_t)U;
+    const bool live = u0 + i * TG < U;
     const bool short_row = live && m.n > 0u && m.n <= (uint32_t)LONG_ROW;
     if (l == 0) {
       *reinterpret_cast<float4*>(sl) =
@@ -868,7 +877,9 @@ __global__ void __launch_bounds__(STAGE_THREADS, CPL == 1 ? GBA_STAGE_MINB : (CP
     commit();
   }
 
-  for (int64_t i = 0; gw * G + i * TG < (int64_t)U; ++i) {
+  // every group of the warp runs the same iterations (the loop holds __syncwarp)
+  const uint32_t uw = gw * (uint32_t)G;
+  for (uint32_t i = 0; uw + i * TG < U; ++i) {
     asm volatile("cp.async.wait_group %0;" ::"n"(STAGE_P - 1) : "memory");
     __syncwarp();
     // ---- apply row i from its data slot: its kept gradients summed in sorted order
