@@ -474,7 +474,8 @@ def run_gba(args):
         cpu_batches = [[{"token": m["token"], "local_batch": m["local_batch"],
                          "ids": [x.cpu() for x in m["ids"]], "rows": [x.cpu() for x in m["rows"]],
                          "dense": m["dense"].cpu()} for m in b] for b in batches]
-        sps, sample = oracle_rate(cfg, cpu_batches, 1, args.cpu_steps)
+        # the same warm-up as the reference arm, so both report one number
+        sps, sample = oracle_rate(cfg, cpu_batches, args.warmup, args.cpu_steps)
         cpu = {"value": sps, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": sample}
         del cpu_batches
 
@@ -531,7 +532,7 @@ def main():
     ap.add_argument("--shape-dense", type=int, default=None,
                     help="dense parameters (profiling case of the same shape)")
     ap.add_argument("--cpu-steps", type=int, default=3,
-                    help="oracle steps timed for the cpu_baseline leg (after one warm-up step)")
+                    help="oracle steps timed for the cpu_baseline leg (after --warmup untimed steps)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
