@@ -74,7 +74,8 @@ typedef struct {
 } gba_opt_desc;
 
 /* One embedding table: rows x dim float32 weights plus optimizer state and a
- * per-row step tag (Alg. 2 "global step of appearance tagged to each ID"). */
+ * per-row step tag (Alg. 2: each ID carries the global step at which it was last
+ * updated). */
 typedef struct {
   int64_t rows;            /* >= 1; the sum of rows over all tables must be < 2^32 */
   int32_t dim;             /* 1 .. 256 */
@@ -88,8 +89,8 @@ typedef struct {
  *   row_staleness 0: rows use the row's step tag as the reference (Alg. 2),
  *                 1: rows use the current step k, like the dense gradient.
  *   sparse_denominator 0: divide a row's kept sum by the number of messages in
- *                 the global batch that contain the row (Alg. 2 "workers that
- *                 encountered the particular ID"), 1: by the kept ones, 2: by M.
+ *                 the global batch that contain the row (Alg. 2: the workers
+ *                 whose batches held the ID), 1: by the kept ones, 2: by M.
  *   decay 0: a kept gradient weighs 1 (Eq. (1) as printed);
  *         1: a kept gradient of staleness s weighs lambda^s (Sec. 4.1 allows
  *            other decay strategies; lambda^s is s products in double, rounded
@@ -192,8 +193,8 @@ gba_status gba_push_ref(gba_handle* h, int64_t token, const gba_sparse_grad* per
 
 /*
  * gba_try_apply - if the buffered local batches reach the global batch, pop the
- * oldest messages that do (Alg. 2: "pop N_a gradients"), enqueue one global
- * step on the stream and return 1; otherwise return 0.  The step:
+ * oldest messages that do (Alg. 2 takes N_a gradients off the buffer), enqueue
+ * one global step on the stream and return 1; otherwise return 0.  The step:
  *   Eq. (1) weights per message; rows deduplicated by id (radix sort);
  *   per row: decay by the row's tag vs the token, sum of kept gradients divided
  *   by the denominator, optimizer, tag := k + 1 (rows with no kept gradient are

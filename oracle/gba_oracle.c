@@ -16,7 +16,7 @@
  *   - dense: weighted sum over the popped gradients divided by N_a
  *                                                   Alg. 2 (push responding)
  *   - embeddings: per-ID step tags, decay by tag vs token, weighted sum divided
- *     by the number of workers that encountered the ID
+ *     by the number of workers whose batches contained the ID
  *                                                   Alg. 2 (push responding)
  *   - update form w <- w - eta * v, v = (1/M) sum g  Appendix A, proof of Thm 1
  *   - optimizers Adagrad / Adam                      Table 1
@@ -347,7 +347,7 @@ int gbao_step(int64_t k, const gbao_rule* rule, int32_t M, const int64_t* tokens
       bc1 = adam_bias_correction(tb->opt.beta1, t_step);
       bc2 = adam_bias_correction(tb->opt.beta2, t_step);
     }
-    /* Weighted sum divided by the number of workers that encountered the ID;
+    /* Weighted sum divided by the number of workers whose batches contained the ID;
      * rows whose gradients were all excluded take no step and keep their tag. */
     for (int64_t r = 0; r < nt; ++r) {
       if (cnt[r] > 0) st.rows_touched++;

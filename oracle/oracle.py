@@ -6,7 +6,7 @@ imports this module and shares no code with ``gba_oracle.c``.
 
 ``OracleGBA`` is the parameter server of Alg. 2 reduced to one process: a FIFO
 gradient buffer that pops the shortest prefix of messages whose local batches
-reach the global batch (Sec. 4.1, "at least N_a gradients ... pop N_a"), then
+reach the global batch (Sec. 4.1: apply once N_a gradients are buffered), then
 runs one global step of ``gba_oracle.c`` on them.  State is kept only for a
 tracked set of rows per table and of dense elements; rows are independent of
 one another, so any subset evolves exactly as it would in the full model.

@@ -1,6 +1,6 @@
-// Pull responding (Alg. 2): "look up the embedding tables based on the IDs"
-// and send the parameters back to the worker.  One kernel gathers the current
-// rows of one table for a list of ids into a caller buffer.
+// Pull responding (Alg. 2): the PS answers a worker with the current embedding
+// rows of the IDs it asks for.  One kernel gathers the current rows of one
+// table for a list of ids into a caller buffer.
 //
 // Layout: L lanes per row (the smallest power of two >= d/4, at most 32), each
 // lane moving 16-byte pieces when d is a multiple of 4 (rows are then 16-byte

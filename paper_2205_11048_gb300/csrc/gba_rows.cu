@@ -1,7 +1,7 @@
 // K3 + K4 of the GBA aggregate-and-apply step: per unique row of the sorted
 // occurrence array, decay each occurrence by the row's step tag against its
 // message's token (Eq. (1); Alg. 2, push responding), sum the kept gradient
-// rows, divide by the number of messages that encountered the row, apply the
+// rows, divide by the number of messages whose ids include the row, apply the
 // optimizer to the row and its state in place, and set the row's tag to k + 1.
 //
 // Three kernels per table:
@@ -103,7 +103,7 @@ __device__ __forceinline__ int message_of(const uint32_t* off, int M, uint32_t x
   return message_of_any(off, M, x);
 }
 
-// Denominator of a row's weighted sum (Alg. 2: messages that encountered the
+// Denominator of a row's weighted sum (Alg. 2: messages whose ids include the
 // row; or the messages whose occurrence was kept; or all M messages).
 __device__ __forceinline__ float row_denominator(int mode, uint32_t c_all, uint32_t c_kept, int M) {
   const uint32_t den = mode == 0 ? c_all : (mode == 1 ? c_kept : (uint32_t)M);
