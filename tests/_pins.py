@@ -241,7 +241,8 @@ def pin_sync_closed_form(L, seed=3):
         ghat = np.zeros((V, d))
         ghat[touched] = S[touched] / c[touched, None]
         a1 = a0 + ghat**2
-        w1 = np.where(touched[:, None], w0 - 0.05 * ghat / np.sqrt(a1), w0)
+        with np.errstate(divide="ignore", invalid="ignore"):  # untouched rows are not used
+            w1 = np.where(touched[:, None], w0 - 0.05 * ghat / np.sqrt(a1), w0)
         a1 = np.where(touched[:, None], a1, a0)
         gbar = np.mean(np.stack([m.dense.astype(np.float64) for m in msgs]), axis=0)
         da1 = da0 + gbar**2
@@ -541,9 +542,37 @@ def pin_hash_ids(L, seed=41):
         raise AssertionError("the reserved id was accepted")
 
 
+def pin_modulo_ids(L, seed=51):
+    """MODULO tables (hashing trick): a table fed arbitrary int64 ids, negative
+    ones included, evolves bit for bit as a DIRECT table fed the residues of
+    the ids read as unsigned 64-bit integers, computed here with Python's
+    exact integer arithmetic."""
+    rng = np.random.default_rng(seed)
+    V, d, D, M = 7, 2, 3, 3
+    for kind in (O.ADAGRAD, O.ADAM):
+        mod = O.OracleGBA([O.TableSpec(V, d, O.OptSpec(kind, 0.03), id_mode=1)], D,
+                          O.OptSpec(kind, 0.01), M, iota=1, seed=4, library=L)
+        direct = O.OracleGBA([O.TableSpec(V, d, O.OptSpec(kind, 0.03))], D,
+                             O.OptSpec(kind, 0.01), M, iota=1, seed=4, library=L)
+        for s in range(3):
+            for m in range(M):
+                n = int(rng.integers(0, 6))
+                ids = rng.integers(-2**63, 2**63 - 1, n, dtype=np.int64)
+                res = np.array([(int(x) % 2**64) % V for x in ids], np.int64)
+                rows = (rng.standard_normal((n, d)) * .5).astype(np.float32)
+                dense = (rng.standard_normal(D) * .5).astype(np.float32)
+                tok = max(0, s - int(rng.integers(0, 3)))
+                mod.push(O.Message(tok, 1, [ids], [rows], dense))
+                direct.push(O.Message(tok, 1, [res], [rows], dense))
+            assert mod.try_apply() == 1 and direct.try_apply() == 1
+        assert mod.tables[0].w.tobytes() == direct.tables[0].w.tobytes()
+        assert mod.tables[0].s0.tobytes() == direct.tables[0].s0.tobytes()
+        assert mod.tables[0].ver.tolist() == direct.tables[0].ver.tolist()
+
+
 ALL_PINS = [pin_hand_adagrad, pin_hand_rule_options, pin_hand_decay_variants,
             pin_decay_special_cases, pin_hand_adam, pin_sync_closed_form, pin_decay_boundary,
-            pin_fifo_prefix, pin_order_invariance, pin_brute_force, pin_hash_ids]
+            pin_fifo_prefix, pin_order_invariance, pin_brute_force, pin_hash_ids, pin_modulo_ids]
 
 
 def pin_init_published(L):

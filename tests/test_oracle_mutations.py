@@ -61,6 +61,13 @@ MUTATIONS = [
      "if (m > M - rule->drop_latest) return 0.0f;", 0),
     ("hash-reserved-id-accepted", "if (id == INT64_MIN) { err = 1; continue; }",
      "if (id == INT64_MIN) { x = id; }", 0),
+    ("adam-eps-inside-sqrt", "float den = sqrtf(vhat) + o->eps;", "float den = sqrtf(vhat + o->eps);", 0),
+    ("adam-no-bias-correction", "float mhat = mn / bc1;", "float mhat = mn;", 0),
+    ("tag-set-to-k", "tb->ver[r] = k + 1;", "tb->ver[r] = k;", 0),
+    ("staleness-not-clamped", "return s < 0 ? 0 : s;", "return s;", 0),
+    ("adagrad-init-zero", "tb->s0[i] = tb->opt.init_acc;", "tb->s0[i] = 0.0f;", 0),
+    ("modulo-signed-residue", "x = (int64_t)((uint64_t)id % (uint64_t)tb->V);",
+     "x = id % tb->V; if (x < 0) x += tb->V;", 0),
     ("hash-ids-folded", "  /* the reserved id */\n          x = id;",
      "  /* the reserved id */\n          x = (int64_t)((uint64_t)id % (uint64_t)tb->V);", 0),
 ]
