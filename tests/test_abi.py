@@ -87,6 +87,22 @@ def test_null_handle_calls_are_safe(L):
     L.gba_destroy(None)
     assert L.gba_last_error(None) == b""
     assert L.gba_selftest_wait_timeout(-1, None) == B.GBA_E_ARG
+    # every other entry point that takes a handle refuses a NULL one
+    for call in (lambda: L.gba_push_ref(None, 0, None, None, 1),
+                 lambda: L.gba_join(None), lambda: L.gba_set_overlap(None, 1),
+                 lambda: L.gba_set_eager_dense(None, 1), lambda: L.gba_set_timing(None, 1),
+                 lambda: L.gba_set_debug(None, 1), lambda: L.gba_kernel_times(None, None),
+                 lambda: L.gba_get_table(None, 0, None, None, None, None),
+                 lambda: L.gba_get_dense(None, None, None, None),
+                 lambda: L.gba_table_capacity(None, 0, None),
+                 lambda: L.gba_lookup_rows(None, 0, None, 0, None),
+                 lambda: L.gba_pull(None, 0, None, 0, None),
+                 lambda: L.gba_debug_segments(None, 0, None, None, None, None, None),
+                 lambda: L.gba_debug_sorted(None, 0, None, None, None),
+                 lambda: L.gba_debug_keep(None, 0, None, None),
+                 lambda: L.gba_debug_set_wait_limit(None, 0),
+                 lambda: L.gba_debug_withhold_dense_copies(None, 1)):
+        assert call() == B.GBA_E_ARG
 
 
 def test_create_without_gpu_fails_cleanly(L):
