@@ -283,8 +283,9 @@ def test_varying_local_batches_overshoot():
 
 
 def test_hot_row_spanning_many_warps():
-    """One row with 200K occurrences in a step: its partial sums span hundreds
-    of reduction windows and are merged by the cross-window kernel."""
+    """One row with 200K occurrences in a step: its kept occurrences fill
+    hundreds of chunks, summed by different warps and merged in chunk order by
+    the warp that finishes the last one."""
     gen = torch.Generator(device="cuda").manual_seed(1)
     cfg = cfg_of([(5000, 16, 0, 1)], D=4, G=4, iota=2)
     steps = []
@@ -297,6 +298,41 @@ def test_hot_row_spanning_many_warps():
             batch.append(msg(max(0, k - m % 3), [ids.cpu().numpy()], [16], 4))
         steps.append(batch)
     run_custom(cfg, steps, max_ids=60_000)
+
+
+@pytest.mark.parametrize("dim", [64, 12])
+@pytest.mark.parametrize("rule", [None, dict(iota=2, decay=1, lam=0.5)])
+def test_kept_count_boundaries_of_the_row_kernels(dim, rule):
+    """Rows whose kept occurrences sit on each side of the row kernels' limits
+    -- 4 (short rows), 32 (one lane group per row) and multiples of the
+    128-occurrence chunks -- against the oracle: all messages kept, stale
+    messages dropped, and geometric weights."""
+    counts = [1, 2, 4, 5, 6, 31, 32, 33, 64, 127, 128, 129, 130, 255, 256, 257, 300]
+    V, M, D = len(counts) + 3, 8, 37
+    iota = (rule or {}).get("iota", 1)
+    cfg = cfg_of([(V, dim, 0, 0)], D=D, G=M, iota=iota)
+    rng = np.random.default_rng(dim)
+
+    def batch(k, stale):
+        per = [[] for _ in range(M)]
+        for r, c in enumerate(counts):
+            for _ in range(c):
+                per[int(rng.integers(0, M))].append(r)
+        toks = [max(0, k - 3) if m in stale else k for m in range(M)]
+        return [msg(toks[m], [np.array(per[m], np.int64)], [dim], D,
+                    gen=torch.Generator(device="cuda").manual_seed(100 * k + m)) for m in range(M)]
+
+    steps = [batch(0, []), batch(1, []), batch(2, [1, 5]), batch(3, [0]), batch(4, [])]
+    run_custom(cfg, steps, rule=rule)
+
+
+@pytest.mark.parametrize("D", [2048 * 152 * 2 + 6, 2048 * 152 * 3 * 2 + 2048 + 6])
+def test_dense_tiles_over_many_ctas(D):
+    """Dense sizes that give some CTAs more tiles than others, a short last
+    tile and a ragged tail of 2 elements, every element against the oracle."""
+    cfg = cfg_of([], D=D, G=3)
+    run_custom(cfg, [[msg(0, [], [], D), msg(0, [], [], D), msg(0, [], [], D)],
+                     [msg(1, [], [], D), msg(0, [], [], D), msg(1, [], [], D)]], by_ref=True)
 
 
 def test_dense_only_and_tables_only():
@@ -315,9 +351,10 @@ def test_dense_sizes(D):
 
 
 def test_ragged_sort_sizes():
-    """Step sizes around the sort tile (4096) and the segment round (64)."""
+    """Step sizes around the sort and segment-scan tiles (2048 positions) and
+    the classification tiles (2048 row records)."""
     rng = np.random.default_rng(2)
-    for n in (1, 63, 64, 65, 4095, 4096, 4097, 12289):
+    for n in (1, 63, 64, 65, 2047, 2048, 2049, 4095, 4096, 4097, 12289):
         cfg = cfg_of([(70_000, 8, 0, 0)], D=4, G=1)
         run_custom(cfg, [[msg(0, [rng.integers(0, 70_000, n)], [8], 4)]], max_ids=n)
 
