@@ -300,7 +300,7 @@ def test_hot_row_spanning_many_warps():
     run_custom(cfg, steps, max_ids=60_000)
 
 
-@pytest.mark.parametrize("dim", [64, 12])
+@pytest.mark.parametrize("dim", [64, 12, 14])  # 14: the register path (not a multiple of 4)
 @pytest.mark.parametrize("rule", [None, dict(iota=2, decay=1, lam=0.5)])
 def test_kept_count_boundaries_of_the_row_kernels(dim, rule):
     """Rows whose kept occurrences sit on each side of the row kernels' limits
